@@ -1,0 +1,97 @@
+// Internal host-side launchers shared by the library's translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace cora {
+struct Top1;
+}
+
+// Partial Eq. 1 state of one row over part of the vocabulary (see Top1 in
+// cora_device.cuh): running max logit, sum of exp(logit - max), lowest index
+// of the max.  Layout of a partial array: [n_parts][rows].
+struct Top1Part {
+  float m;
+  float s;
+  int32_t idx;
+};
+
+// Gate launch parameters for the session path (one warp per sequence).
+struct SessionGateArgs {
+  const Top1Part* parts;  // [n_parts][B * BL]
+  int n_parts;
+  int32_t* ctrl;          // [B][4] {block, step, passes, finished}
+  int32_t* tokens;        // [B][S]
+  uint8_t* state;         // [B][G]
+  int32_t* persist;       // [B][BL]
+  int32_t* prev;          // [B][BL]
+  float* conf;            // [B][BL]
+  int32_t* argmax;        // [B][BL]
+  uint8_t* unmask;        // [B][BL]
+  uint8_t* accept;        // [B][BL]
+  uint8_t* all_done;      // [1]
+  int* err;
+  int B, S, P, G, BL, T;
+  float tau;
+  int K;
+};
+
+void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_t start, float scale,
+                              cudaStream_t st);
+void launch_embed(const int32_t* tokens, const uint16_t* embed, float* h, int M, int d, cudaStream_t st);
+void launch_rmsnorm(const float* x, const uint16_t* w, uint16_t* out, int M, int d, float eps, cudaStream_t st);
+void launch_final_norm_rows(const float* h, const uint16_t* w, const int32_t* ctrl, uint16_t* out, int B, int S,
+                            int P, int BL, int n_blocks, int d, float eps, cudaStream_t st);
+
+// Eq. 1 partials from materialised bf16 logits [rows, V]: grid (n_chunks, rows).
+int reduce_top1_parts_count(int rows, int V, int num_sms);
+void launch_reduce_top1_parts(const uint16_t* logits, int rows, int V, int n_chunks, Top1Part* parts,
+                              cudaStream_t st);
+void launch_combine_top1(const Top1Part* parts, int n_parts, int rows, float* conf, int32_t* argmax,
+                         cudaStream_t st);
+void launch_gate_transfer(const Top1Part* parts, int n_parts, const float* conf_in, const int32_t* argmax_in,
+                          float* conf_out, int32_t* argmax_out, int32_t* prev, int32_t* persist, uint8_t* state,
+                          int32_t* tokens, int B, int R, int k, float tau, int K, uint8_t* unmask, uint8_t* accept,
+                          uint8_t* done, cudaStream_t st);
+void launch_session_gate(const SessionGateArgs& a, cudaStream_t st);
+
+// GEMM (tcgen05).  Epilogue parameters.
+struct GemmEpilogue {
+  void* C;
+  int ldc;
+  int mode;             // CORA_EPI_*
+  const float* rope;    // [seq][head_dim/2][2]
+  int seq;
+  int head_dim;
+  int rope_cols;
+};
+
+// Tensor-map encoder (driver entry point fetched at runtime).
+bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
+                       uint32_t box_rows, uint32_t box_cols);
+
+int gemm_block_n(int N, int mode);
+cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K,
+                        const GemmEpilogue& ep, int* err, int num_sms, cudaStream_t st);
+
+// Fused LM head + Eq. 1 partials: x [R, d] (tensor map box rows = n_pad),
+// W [V, d].  Writes parts [grid][R]; returns the number of parts used.
+int lm_head_parts_count(int V, int num_sms);
+int lm_head_npad(int R);
+cudaError_t launch_lm_head_top1(const CUtensorMap& tmW, const CUtensorMap& tmX, int R, int V, int d,
+                                Top1Part* parts, int n_parts, int* err, cudaStream_t st);
+
+// Shared-memory attributes of the big-smem kernels (call once per device,
+// outside stream capture).
+cudaError_t gemm_prepare();
+cudaError_t lm_head_prepare();
+cudaError_t attention_prepare();
+
+void launch_session_init(int32_t* tokens, const int32_t* prompt, uint8_t* state, int32_t* persist, int32_t* prev,
+                         int32_t* ctrl, int32_t* status, int B, int P, int S, int G, int BL, int mask_id,
+                         cudaStream_t st);
+
+// Attention.
+void launch_attention(const uint16_t* qkv, uint16_t* out, int B, int S, int Hq, int Hkv, int hd, cudaStream_t st);

@@ -1,0 +1,719 @@
+// C ABI of the CORA-Diff library: model and session objects, the per-step
+// CUDA graph (dense pass -> active-row LM head + Eq. 1 -> gate), the decode
+// loop, and the standalone kernel entry points.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <cmath>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/cora.h"
+#include "cora_kernels.h"
+
+// ------------------------------------------------------------------ errors
+static thread_local std::string g_last_error;
+
+static int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
+#define CK(call)                                                                        \
+  do {                                                                                  \
+    cudaError_t e_ = (call);                                                            \
+    if (e_ != cudaSuccess) {                                                            \
+      return fail(e_ == cudaErrorMemoryAllocation ? CORA_ENOMEM : CORA_ECUDA, "%s: %s", \
+                  #call, cudaGetErrorString(e_));                                       \
+    }                                                                                   \
+  } while (0)
+
+#define REQUIRE(cond, ...)                     \
+  do {                                         \
+    if (!(cond)) return fail(CORA_EINVAL, __VA_ARGS__); \
+  } while (0)
+
+extern "C" const char* cora_last_error(void) { return g_last_error.c_str(); }
+extern "C" int cora_version(void) { return 100; }
+
+// --------------------------------------------------------- device context
+namespace {
+
+struct DeviceCtx {
+  bool ready = false;
+  bool prepared = false;
+  int num_sms = 0;
+  int* err = nullptr;          // device error word for standalone ops
+  void* scratch = nullptr;     // partials for standalone reductions
+  size_t scratch_bytes = 0;
+};
+
+std::mutex g_mu;
+DeviceCtx g_dev[16];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int device_ctx(DeviceCtx** out) {
+  int dev = 0;
+  CK(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= 16) return fail(CORA_EINVAL, "device index %d unsupported", dev);
+  std::lock_guard<std::mutex> lk(g_mu);
+  DeviceCtx& c = g_dev[dev];
+  if (!c.ready) {
+    CK(cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, dev));
+    CK(cudaMalloc(&c.err, sizeof(int)));
+    CK(cudaMemset(c.err, 0, sizeof(int)));
+    if (!g_encode) {
+      cudaDriverEntryPointQueryResult q;
+      void* fn = nullptr;
+      CK(cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q));
+      if (q != cudaDriverEntryPointSuccess || !fn) return fail(CORA_ECUDA, "cuTensorMapEncodeTiled unavailable");
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    c.ready = true;
+  }
+  *out = &c;
+  return CORA_OK;
+}
+
+int scratch_reserve(DeviceCtx* c, size_t bytes, void** out) {
+  if (c->scratch_bytes < bytes) {
+    if (c->scratch) CK(cudaFree(c->scratch));
+    c->scratch = nullptr;
+    c->scratch_bytes = 0;
+    CK(cudaMalloc(&c->scratch, bytes));
+    c->scratch_bytes = bytes;
+  }
+  *out = c->scratch;
+  return CORA_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
+                       uint32_t box_rows, uint32_t box_cols) {
+  if (!g_encode) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {row_stride_bytes};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+// Sets the shared-memory attributes of every kernel instance, once per device.
+static int kernels_prepare() {
+  DeviceCtx* dc = nullptr;
+  int rc = device_ctx(&dc);
+  if (rc) return rc;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if (!dc->prepared) {
+    CK(gemm_prepare());
+    CK(lm_head_prepare());
+    CK(attention_prepare());
+    dc->prepared = true;
+  }
+  return CORA_OK;
+}
+
+// ------------------------------------------------------------------ model
+struct cora_model {
+  cora_model_config cfg{};
+  int f_pad = 0;   // ffn rounded up to a multiple of 128
+  int n_qkv = 0;   // (n_heads + 2 n_kv_heads) * head_dim
+  int num_sms = 0;
+  uint16_t* embed = nullptr;
+  uint16_t* head = nullptr;
+  uint16_t* final_norm = nullptr;
+  std::vector<uint16_t*> attn_norm, ffn_norm, wqkv, wo, wgu, wdown;
+  std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
+  CUtensorMap tm_head{};
+  std::vector<void*> allocs;
+  cora_session* cached = nullptr;
+};
+
+static int model_alloc(cora_model* m, size_t bytes, uint16_t** out) {
+  void* p = nullptr;
+  CK(cudaMalloc(&p, bytes));
+  m->allocs.push_back(p);
+  *out = static_cast<uint16_t*>(p);
+  return CORA_OK;
+}
+
+static void model_free(cora_model* m) {
+  for (void* p : m->allocs) cudaFree(p);
+  m->allocs.clear();
+}
+
+static int copy_rows(uint16_t* dst, const uint16_t* src, size_t rows, size_t cols) {
+  CK(cudaMemcpy(dst, src, rows * cols * 2, cudaMemcpyDefault));
+  return CORA_OK;
+}
+
+extern "C" int cora_model_destroy(cora_model* m);
+extern "C" int cora_session_destroy(cora_session* s);
+
+extern "C" int cora_model_create(const cora_model_config* cfg, const cora_weights* w, cora_model** out) {
+  REQUIRE(cfg && w && out, "cora_model_create: NULL argument");
+  const cora_model_config c = *cfg;
+  REQUIRE(c.n_layers >= 1 && c.d_model >= 128 && c.d_model % 128 == 0, "d_model must be a positive multiple of 128");
+  REQUIRE(c.head_dim == 64 || c.head_dim == 128, "head_dim must be 64 or 128");
+  REQUIRE(c.n_heads >= 1 && c.n_kv_heads >= 1 && c.n_heads % c.n_kv_heads == 0, "n_heads %% n_kv_heads != 0");
+  REQUIRE((c.n_heads * c.head_dim) % 64 == 0, "n_heads * head_dim must be a multiple of 64");
+  REQUIRE(((c.n_heads + 2 * c.n_kv_heads) * c.head_dim) % 128 == 0,
+          "(n_heads + 2 n_kv_heads) * head_dim must be a multiple of 128");
+  REQUIRE(c.ffn >= 1 && c.vocab >= 2 && c.mask_id >= 0 && c.mask_id < c.vocab, "bad ffn/vocab/mask_id");
+  REQUIRE(c.norm_eps >= 0.f && c.rope_theta > 0.f, "bad norm_eps/rope_theta");
+  REQUIRE(w->embed && w->lm_head && w->wq && w->wk && w->wv && w->wo && w->w_gate && w->w_up && w->w_down,
+          "cora_model_create: NULL weight");
+  for (int l = 0; l < c.n_layers; ++l)
+    REQUIRE(w->wq[l] && w->wk[l] && w->wv[l] && w->wo[l] && w->w_gate[l] && w->w_up[l] && w->w_down[l],
+            "cora_model_create: NULL weight in layer %d", l);
+
+  DeviceCtx* dc = nullptr;
+  int rc = device_ctx(&dc);
+  if (rc) return rc;
+  if ((rc = kernels_prepare())) return rc;
+
+  cora_model* m = new cora_model();
+  m->cfg = c;
+  m->num_sms = dc->num_sms;
+  m->f_pad = (c.ffn + 127) / 128 * 128;
+  m->n_qkv = (c.n_heads + 2 * c.n_kv_heads) * c.head_dim;
+  const size_t d = c.d_model, hq = size_t(c.n_heads) * c.head_dim, hkv = size_t(c.n_kv_heads) * c.head_dim;
+  const size_t F = c.ffn, FP = m->f_pad;
+
+#define MK(call)          \
+  do {                    \
+    int r_ = (call);      \
+    if (r_) {             \
+      cora_model_destroy(m); \
+      return r_;          \
+    }                     \
+  } while (0)
+
+  MK(model_alloc(m, size_t(c.vocab) * d * 2, &m->embed));
+  MK(copy_rows(m->embed, w->embed, c.vocab, d));
+  MK(model_alloc(m, size_t(c.vocab) * d * 2, &m->head));
+  MK(copy_rows(m->head, w->lm_head, c.vocab, d));
+  if (w->final_norm) {
+    MK(model_alloc(m, d * 2, &m->final_norm));
+    MK(copy_rows(m->final_norm, w->final_norm, 1, d));
+  }
+  for (int l = 0; l < c.n_layers; ++l) {
+    uint16_t *an = nullptr, *fn = nullptr, *qkv, *wo, *gu, *dn;
+    if (w->attn_norm && w->attn_norm[l]) {
+      MK(model_alloc(m, d * 2, &an));
+      MK(copy_rows(an, w->attn_norm[l], 1, d));
+    }
+    if (w->ffn_norm && w->ffn_norm[l]) {
+      MK(model_alloc(m, d * 2, &fn));
+      MK(copy_rows(fn, w->ffn_norm[l], 1, d));
+    }
+    MK(model_alloc(m, size_t(m->n_qkv) * d * 2, &qkv));
+    MK(copy_rows(qkv, w->wq[l], hq, d));
+    MK(copy_rows(qkv + hq * d, w->wk[l], hkv, d));
+    MK(copy_rows(qkv + (hq + hkv) * d, w->wv[l], hkv, d));
+    MK(model_alloc(m, d * hq * 2, &wo));
+    MK(copy_rows(wo, w->wo[l], d, hq));
+    // gate/up interleaved in groups of 128 rows: [gate 128 | up 128] per group.
+    MK(model_alloc(m, 2 * FP * d * 2, &gu));
+    if (FP != F) CK(cudaMemset(gu, 0, 2 * FP * d * 2));
+    for (size_t g0 = 0; g0 < F; g0 += 128) {
+      const size_t n = (F - g0) < 128 ? (F - g0) : 128;
+      MK(copy_rows(gu + (2 * g0) * d, w->w_gate[l] + g0 * d, n, d));
+      MK(copy_rows(gu + (2 * g0 + 128) * d, w->w_up[l] + g0 * d, n, d));
+    }
+    MK(model_alloc(m, d * FP * 2, &dn));
+    if (FP != F) CK(cudaMemset(dn, 0, d * FP * 2));
+    CK(cudaMemcpy2D(dn, FP * 2, w->w_down[l], F * 2, F * 2, d, cudaMemcpyDefault));
+    m->attn_norm.push_back(an);
+    m->ffn_norm.push_back(fn);
+    m->wqkv.push_back(qkv);
+    m->wo.push_back(wo);
+    m->wgu.push_back(gu);
+    m->wdown.push_back(dn);
+    CUtensorMap t1, t2, t3, t4;
+    bool ok = make_tmap_bf16_2d(&t1, qkv, m->n_qkv, d, d * 2, gemm_block_n(m->n_qkv, CORA_EPI_ROPE_BF16), 64) &&
+              make_tmap_bf16_2d(&t2, wo, d, hq, hq * 2, gemm_block_n(int(d), CORA_EPI_RESID_F32), 64) &&
+              make_tmap_bf16_2d(&t3, gu, 2 * FP, d, d * 2, gemm_block_n(int(2 * FP), CORA_EPI_SWIGLU), 64) &&
+              make_tmap_bf16_2d(&t4, dn, d, FP, FP * 2, gemm_block_n(int(d), CORA_EPI_RESID_F32), 64);
+    if (!ok) {
+      cora_model_destroy(m);
+      return fail(CORA_ECUDA, "tensor map encoding failed (layer %d)", l);
+    }
+    m->tm_qkv.push_back(t1);
+    m->tm_o.push_back(t2);
+    m->tm_gu.push_back(t3);
+    m->tm_down.push_back(t4);
+  }
+  if (!make_tmap_bf16_2d(&m->tm_head, m->head, c.vocab, d, d * 2, 128, 64)) {
+    cora_model_destroy(m);
+    return fail(CORA_ECUDA, "tensor map encoding failed (lm head)");
+  }
+#undef MK
+  CK(cudaDeviceSynchronize());
+  *out = m;
+  return CORA_OK;
+}
+
+// ---------------------------------------------------------------- session
+struct cora_session {
+  cora_model* m = nullptr;
+  int B = 0, P = 0, G = 0, S = 0, BL = 0, T = 0, n_blocks = 0, M = 0, R = 0;
+  float tau = 0.f;
+  int K = 0;
+  cudaStream_t stream = nullptr;
+  std::vector<void*> allocs;
+  int32_t* prompt = nullptr;   // [B, P] copy used by reset
+  int32_t* tokens = nullptr;   // [B, S]
+  float* h = nullptr;          // [M, d] residual stream
+  uint16_t* xn = nullptr;      // [M, d] normalised activations
+  uint16_t* qkv = nullptr;     // [M, n_qkv]
+  uint16_t* attn = nullptr;    // [M, Hq*hd]
+  uint16_t* act = nullptr;     // [M, f_pad]
+  uint16_t* xf = nullptr;      // [R, d] final-normed active rows
+  float* rope = nullptr;       // [S, hd/2, 2]
+  Top1Part* parts = nullptr;   // [n_parts, R]
+  int n_parts = 0;
+  int32_t* ctrl = nullptr;     // [B, 4]
+  uint8_t* state = nullptr;    // [B, G]
+  int32_t* persist = nullptr;  // [B, BL]
+  int32_t* prev = nullptr;     // [B, BL]
+  float* conf = nullptr;       // [B, BL]
+  int32_t* argmax = nullptr;   // [B, BL]
+  uint8_t* unmask = nullptr;   // [B, BL]
+  uint8_t* accept = nullptr;   // [B, BL]
+  int32_t* status = nullptr;   // device {all_done (byte 0), error word}
+  int32_t* status_h = nullptr; // pinned host copy
+  CUtensorMap tm_xn{}, tm_attn{}, tm_act{}, tm_xf{};
+  cudaGraphExec_t graph = nullptr;
+  int64_t batched_passes = 0;
+  bool finished = false;
+};
+
+template <typename T>
+static int sess_alloc(cora_session* s, size_t count, T** out) {
+  void* p = nullptr;
+  CK(cudaMalloc(&p, count * sizeof(T) < 16 ? 16 : count * sizeof(T)));
+  s->allocs.push_back(p);
+  *out = static_cast<T*>(p);
+  return CORA_OK;
+}
+
+static int enqueue_step(cora_session* s) {
+  cora_model* m = s->m;
+  const cora_model_config& c = m->cfg;
+  const int d = c.d_model, M = s->M;
+  int* err = s->status + 1;
+  cudaStream_t st = s->stream;
+  launch_embed(s->tokens, m->embed, s->h, M, d, st);
+  for (int l = 0; l < c.n_layers; ++l) {
+    launch_rmsnorm(s->h, m->attn_norm[l], s->xn, M, d, c.norm_eps, st);
+    GemmEpilogue e1{s->qkv, m->n_qkv, CORA_EPI_ROPE_BF16, s->rope, s->S, c.head_dim,
+                    (c.n_heads + c.n_kv_heads) * c.head_dim};
+    CK(launch_gemm(s->tm_xn, m->tm_qkv[l], M, m->n_qkv, d, e1, err, m->num_sms, st));
+    launch_attention(s->qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, st);
+    GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0};
+    CK(launch_gemm(s->tm_attn, m->tm_o[l], M, d, c.n_heads * c.head_dim, e2, err, m->num_sms, st));
+    launch_rmsnorm(s->h, m->ffn_norm[l], s->xn, M, d, c.norm_eps, st);
+    GemmEpilogue e3{s->act, m->f_pad, CORA_EPI_SWIGLU, nullptr, 0, 0, 0};
+    CK(launch_gemm(s->tm_xn, m->tm_gu[l], M, 2 * m->f_pad, d, e3, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_act, m->tm_down[l], M, d, m->f_pad, e2, err, m->num_sms, st));
+  }
+  launch_final_norm_rows(s->h, m->final_norm, s->ctrl, s->xf, s->B, s->S, s->P, s->BL, s->n_blocks, d, c.norm_eps,
+                         st);
+  CK(launch_lm_head_top1(m->tm_head, s->tm_xf, s->R, c.vocab, d, s->parts, s->n_parts, err, st));
+  SessionGateArgs ga{s->parts, s->n_parts, s->ctrl,  s->tokens, s->state,  s->persist, s->prev,
+                     s->conf,  s->argmax,  s->unmask, s->accept, reinterpret_cast<uint8_t*>(s->status),
+                     err,      s->B,       s->S,      s->P,      s->G,       s->BL,      s->T,
+                     s->tau,   s->K};
+  launch_session_gate(ga, st);
+  CK(cudaGetLastError());
+  CK(cudaMemcpyAsync(s->status_h, s->status, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  return CORA_OK;
+}
+
+extern "C" int cora_session_reset(cora_session* s, const int32_t* prompt) {
+  REQUIRE(s, "cora_session_reset: NULL session");
+  if (prompt && s->P > 0) CK(cudaMemcpyAsync(s->prompt, prompt, size_t(s->B) * s->P * 4, cudaMemcpyDefault, s->stream));
+  launch_session_init(s->tokens, s->prompt, s->state, s->persist, s->prev, s->ctrl, s->status, s->B, s->P, s->S, s->G,
+                      s->BL, s->m->cfg.mask_id, s->stream);
+  CK(cudaGetLastError());
+  CK(cudaStreamSynchronize(s->stream));
+  s->batched_passes = 0;
+  s->finished = false;
+  return CORA_OK;
+}
+
+extern "C" int cora_session_create(cora_model* m, int32_t batch, const int32_t* prompt, int32_t prompt_len,
+                                   int32_t gen_len, int32_t block_len, int32_t steps_per_block, float tau, int32_t K,
+                                   cora_session** out) {
+  REQUIRE(m && out, "cora_session_create: NULL argument");
+  REQUIRE(batch >= 1 && prompt_len >= 0 && gen_len >= 1, "bad batch/prompt_len/gen_len");
+  REQUIRE(block_len >= 1 && block_len <= 32, "block_len must be in [1, 32]");
+  REQUIRE(gen_len % block_len == 0, "gen_len %% block_len != 0");
+  REQUIRE(steps_per_block >= 1, "steps_per_block must be >= 1");
+  REQUIRE(batch * block_len <= 256, "batch * block_len must be <= 256");
+  REQUIRE(prompt_len == 0 || prompt, "NULL prompt");
+  const cora_model_config& c = m->cfg;
+  cora_session* s = new cora_session();
+  s->m = m;
+  s->B = batch;
+  s->P = prompt_len;
+  s->G = gen_len;
+  s->S = prompt_len + gen_len;
+  s->BL = block_len;
+  s->T = steps_per_block;
+  s->n_blocks = gen_len / block_len;
+  s->M = batch * s->S;
+  s->R = batch * block_len;
+  s->tau = tau;
+  s->K = K;
+  const size_t d = c.d_model, M = s->M;
+#define SK(call)              \
+  do {                        \
+    int r_ = (call);          \
+    if (r_) {                 \
+      cora_session_destroy(s); \
+      return r_;              \
+    }                         \
+  } while (0)
+  SK(cudaStreamCreateWithFlags(&s->stream, cudaStreamNonBlocking) == cudaSuccess ? 0
+                                                                               : fail(CORA_ECUDA, "stream create"));
+  SK(sess_alloc(s, size_t(batch) * (prompt_len > 0 ? prompt_len : 1), &s->prompt));
+  SK(sess_alloc(s, M, &s->tokens));
+  SK(sess_alloc(s, M * d, &s->h));
+  SK(sess_alloc(s, M * d, &s->xn));
+  SK(sess_alloc(s, M * size_t(m->n_qkv), &s->qkv));
+  SK(sess_alloc(s, M * size_t(c.n_heads) * c.head_dim, &s->attn));
+  SK(sess_alloc(s, M * size_t(m->f_pad), &s->act));
+  SK(sess_alloc(s, size_t(s->R) * d, &s->xf));
+  SK(sess_alloc(s, size_t(s->S) * c.head_dim, &s->rope));
+  s->n_parts = lm_head_parts_count(c.vocab, m->num_sms);
+  SK(sess_alloc(s, size_t(s->n_parts) * s->R, &s->parts));
+  SK(sess_alloc(s, size_t(batch) * 4, &s->ctrl));
+  SK(sess_alloc(s, size_t(batch) * gen_len, &s->state));
+  SK(sess_alloc(s, size_t(s->R), &s->persist));
+  SK(sess_alloc(s, size_t(s->R), &s->prev));
+  SK(sess_alloc(s, size_t(s->R), &s->conf));
+  SK(sess_alloc(s, size_t(s->R), &s->argmax));
+  SK(sess_alloc(s, size_t(s->R), &s->unmask));
+  SK(sess_alloc(s, size_t(s->R), &s->accept));
+  SK(sess_alloc(s, 4, &s->status));
+  {
+    void* hp = nullptr;
+    if (cudaHostAlloc(&hp, 16, cudaHostAllocDefault) != cudaSuccess) SK(fail(CORA_ENOMEM, "pinned alloc"));
+    s->status_h = static_cast<int32_t*>(hp);
+  }
+  // RoPE table in double precision on the host: angle = pos * theta^(-2j/hd).
+  {
+    const int half = c.head_dim / 2;
+    std::vector<float> tab(size_t(s->S) * half * 2);
+    for (int p = 0; p < s->S; ++p)
+      for (int j = 0; j < half; ++j) {
+        const double ang = double(p) * std::pow(double(c.rope_theta), -2.0 * j / c.head_dim);
+        tab[(size_t(p) * half + j) * 2] = float(std::cos(ang));
+        tab[(size_t(p) * half + j) * 2 + 1] = float(std::sin(ang));
+      }
+    if (cudaMemcpy(s->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+      SK(fail(CORA_ECUDA, "rope table upload"));
+  }
+  const size_t hq = size_t(c.n_heads) * c.head_dim;
+  bool ok = make_tmap_bf16_2d(&s->tm_xn, s->xn, M, d, d * 2, 128, 64) &&
+            make_tmap_bf16_2d(&s->tm_attn, s->attn, M, hq, hq * 2, 128, 64) &&
+            make_tmap_bf16_2d(&s->tm_act, s->act, M, m->f_pad, size_t(m->f_pad) * 2, 128, 64) &&
+            make_tmap_bf16_2d(&s->tm_xf, s->xf, s->R, d, d * 2, lm_head_npad(s->R), 64);
+  if (!ok) SK(fail(CORA_ECUDA, "tensor map encoding failed (session)"));
+  SK(cora_session_reset(s, prompt));
+  // Capture one step (every launch, then the status read-back) as a graph.
+  {
+    cudaGraph_t g = nullptr;
+    if (cudaStreamBeginCapture(s->stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+      SK(fail(CORA_ECUDA, "begin capture"));
+    int rc = enqueue_step(s);
+    cudaError_t ce = cudaStreamEndCapture(s->stream, &g);
+    if (rc) {
+      if (g) cudaGraphDestroy(g);
+      SK(rc);
+    }
+    if (ce != cudaSuccess) SK(fail(CORA_ECUDA, "end capture: %s", cudaGetErrorString(ce)));
+    ce = cudaGraphInstantiate(&s->graph, g, 0);
+    cudaGraphDestroy(g);
+    if (ce != cudaSuccess) SK(fail(CORA_ECUDA, "graph instantiate: %s", cudaGetErrorString(ce)));
+  }
+#undef SK
+  *out = s;
+  return CORA_OK;
+}
+
+extern "C" int cora_session_destroy(cora_session* s) {
+  if (!s) return CORA_OK;
+  if (s->stream) cudaStreamSynchronize(s->stream);
+  if (s->graph) cudaGraphExecDestroy(s->graph);
+  for (void* p : s->allocs) cudaFree(p);
+  if (s->status_h) cudaFreeHost(s->status_h);
+  if (s->stream) cudaStreamDestroy(s->stream);
+  if (s->m && s->m->cached == s) s->m->cached = nullptr;
+  delete s;
+  return CORA_OK;
+}
+
+extern "C" int cora_model_destroy(cora_model* m) {
+  if (!m) return CORA_OK;
+  if (m->cached) cora_session_destroy(m->cached);
+  model_free(m);
+  delete m;
+  return CORA_OK;
+}
+
+extern "C" int cora_denoise_step(cora_session* s, uint8_t* all_done_out) {
+  REQUIRE(s, "cora_denoise_step: NULL session");
+  if (s->finished) return fail(CORA_ESTATE, "every sequence has finished; reset the session");
+  CK(cudaGraphLaunch(s->graph, s->stream));
+  CK(cudaStreamSynchronize(s->stream));
+  s->batched_passes += 1;
+  const int32_t code = s->status_h[1];
+  if (code != 0) return fail(CORA_ETIMEOUT, "device error word 0x%x after step", code);
+  const uint8_t done = reinterpret_cast<const uint8_t*>(s->status_h)[0];
+  s->finished = done != 0;
+  if (all_done_out) *all_done_out = done;
+  return CORA_OK;
+}
+
+extern "C" int cora_session_batched_passes(cora_session* s, int64_t* out) {
+  REQUIRE(s && out, "NULL argument");
+  *out = s->batched_passes;
+  return CORA_OK;
+}
+
+extern "C" int cora_session_read(cora_session* s, int32_t* tokens, uint8_t* state, int32_t* persist, int32_t* prev,
+                                 int32_t* ctrl, float* conf, int32_t* argmax, uint8_t* unmask, uint8_t* accept) {
+  REQUIRE(s, "cora_session_read: NULL session");
+  CK(cudaStreamSynchronize(s->stream));
+  if (tokens) CK(cudaMemcpy(tokens, s->tokens, size_t(s->M) * 4, cudaMemcpyDeviceToHost));
+  if (state) CK(cudaMemcpy(state, s->state, size_t(s->B) * s->G, cudaMemcpyDeviceToHost));
+  if (persist) CK(cudaMemcpy(persist, s->persist, size_t(s->R) * 4, cudaMemcpyDeviceToHost));
+  if (prev) CK(cudaMemcpy(prev, s->prev, size_t(s->R) * 4, cudaMemcpyDeviceToHost));
+  if (ctrl) CK(cudaMemcpy(ctrl, s->ctrl, size_t(s->B) * 16, cudaMemcpyDeviceToHost));
+  if (conf) CK(cudaMemcpy(conf, s->conf, size_t(s->R) * 4, cudaMemcpyDeviceToHost));
+  if (argmax) CK(cudaMemcpy(argmax, s->argmax, size_t(s->R) * 4, cudaMemcpyDeviceToHost));
+  if (unmask) CK(cudaMemcpy(unmask, s->unmask, size_t(s->R), cudaMemcpyDeviceToHost));
+  if (accept) CK(cudaMemcpy(accept, s->accept, size_t(s->R), cudaMemcpyDeviceToHost));
+  return CORA_OK;
+}
+
+extern "C" int cora_session_write(cora_session* s, const int32_t* tokens, const uint8_t* state, const int32_t* persist,
+                                  const int32_t* prev, const int32_t* ctrl) {
+  REQUIRE(s, "cora_session_write: NULL session");
+  CK(cudaStreamSynchronize(s->stream));
+  if (tokens) CK(cudaMemcpy(s->tokens, tokens, size_t(s->M) * 4, cudaMemcpyHostToDevice));
+  if (state) CK(cudaMemcpy(s->state, state, size_t(s->B) * s->G, cudaMemcpyHostToDevice));
+  if (persist) CK(cudaMemcpy(s->persist, persist, size_t(s->R) * 4, cudaMemcpyHostToDevice));
+  if (prev) CK(cudaMemcpy(s->prev, prev, size_t(s->R) * 4, cudaMemcpyHostToDevice));
+  if (ctrl) {
+    CK(cudaMemcpy(s->ctrl, ctrl, size_t(s->B) * 16, cudaMemcpyHostToDevice));
+    bool all = true;
+    for (int b = 0; b < s->B; ++b) all = all && ctrl[b * 4 + 3] != 0;
+    s->finished = all;
+  }
+  return CORA_OK;
+}
+
+extern "C" int cora_generate(cora_model* m, const int32_t* prompt, int32_t B, int32_t P, int32_t gen_len,
+                             int32_t block_len, int32_t steps_per_block, float tau, int32_t K, int32_t* tokens_out,
+                             int64_t* passes_out, int64_t* batched_passes_out) {
+  REQUIRE(m && tokens_out && passes_out, "cora_generate: NULL argument");
+  cora_session* s = m->cached;
+  // tau and K are baked into the captured graph, so they are part of the key.
+  if (s && (s->B != B || s->P != P || s->G != gen_len || s->BL != block_len || s->T != steps_per_block ||
+            s->tau != tau || s->K != K)) {
+    cora_session_destroy(s);
+    s = nullptr;
+  }
+  int rc;
+  if (!s) {
+    rc = cora_session_create(m, B, prompt, P, gen_len, block_len, steps_per_block, tau, K, &s);
+    if (rc) return rc;
+    m->cached = s;
+  } else {
+    rc = cora_session_reset(s, prompt);
+    if (rc) return rc;
+  }
+  const int64_t max_steps = int64_t(s->n_blocks) * s->T;
+  uint8_t done = 0;
+  for (int64_t i = 0; i < max_steps && !done; ++i) {
+    rc = cora_denoise_step(s, &done);
+    if (rc) return rc;
+  }
+  if (!done) return fail(CORA_ESTATE, "decode did not finish within the horizon");
+  CK(cudaMemcpy2D(tokens_out, size_t(gen_len) * 4, s->tokens + P, size_t(s->S) * 4, size_t(gen_len) * 4, B,
+                  cudaMemcpyDeviceToHost));
+  std::vector<int32_t> ctrl(size_t(B) * 4);
+  CK(cudaMemcpy(ctrl.data(), s->ctrl, ctrl.size() * 4, cudaMemcpyDeviceToHost));
+  for (int b = 0; b < B; ++b) passes_out[b] = ctrl[size_t(b) * 4 + 2];
+  if (batched_passes_out) *batched_passes_out = s->batched_passes;
+  return CORA_OK;
+}
+
+// ---------------------------------------------------------- standalone ops
+extern "C" int cora_gate_transfer(const float* conf, const int32_t* argmax, int32_t* prev, int32_t* persist,
+                                  uint8_t* state, int32_t* tokens, int32_t B, int32_t R, int32_t k, float tau,
+                                  int32_t K, uint8_t* unmask, uint8_t* accept, uint8_t* done, void* stream) {
+  REQUIRE(conf && argmax && prev && persist && state && tokens && unmask && accept && done,
+          "cora_gate_transfer: NULL pointer");
+  REQUIRE(B >= 1 && R >= 1 && R <= 32, "cora_gate_transfer: need B >= 1 and 1 <= R <= 32");
+  REQUIRE(k >= 0, "cora_gate_transfer: k must be >= 0");
+  launch_gate_transfer(nullptr, 0, conf, argmax, nullptr, nullptr, prev, persist, state, tokens, B, R, k, tau, K,
+                       unmask, accept, done, static_cast<cudaStream_t>(stream));
+  CK(cudaGetLastError());
+  return CORA_OK;
+}
+
+extern "C" int cora_reduce_top1(const uint16_t* logits, int32_t rows, int32_t V, float* conf, int32_t* argmax,
+                                void* stream) {
+  REQUIRE(logits && conf && argmax, "cora_reduce_top1: NULL pointer");
+  REQUIRE(rows >= 1 && V >= 1, "cora_reduce_top1: rows and V must be >= 1");
+  REQUIRE(V % 8 != 0 || aligned16(logits), "cora_reduce_top1: logits must be 16-byte aligned");
+  DeviceCtx* dc = nullptr;
+  int rc = device_ctx(&dc);
+  if (rc) return rc;
+  const int n = reduce_top1_parts_count(rows, V, dc->num_sms);
+  void* parts = nullptr;
+  rc = scratch_reserve(dc, size_t(n) * rows * sizeof(Top1Part), &parts);
+  if (rc) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  launch_reduce_top1_parts(logits, rows, V, n, static_cast<Top1Part*>(parts), st);
+  launch_combine_top1(static_cast<Top1Part*>(parts), n, rows, conf, argmax, st);
+  CK(cudaGetLastError());
+  return CORA_OK;
+}
+
+extern "C" int cora_reduce_gate(const uint16_t* logits, int32_t B, int32_t R, int32_t V, float* conf, int32_t* argmax,
+                                int32_t* prev, int32_t* persist, uint8_t* state, int32_t* tokens, int32_t k, float tau,
+                                int32_t K, uint8_t* unmask, uint8_t* accept, uint8_t* done, void* stream) {
+  REQUIRE(logits && conf && argmax && prev && persist && state && tokens && unmask && accept && done,
+          "cora_reduce_gate: NULL pointer");
+  REQUIRE(B >= 1 && R >= 1 && R <= 32 && V >= 1 && k >= 0, "cora_reduce_gate: bad shape");
+  REQUIRE(V % 8 != 0 || aligned16(logits), "cora_reduce_gate: logits must be 16-byte aligned");
+  DeviceCtx* dc = nullptr;
+  int rc = device_ctx(&dc);
+  if (rc) return rc;
+  const int rows = B * R;
+  const int n = reduce_top1_parts_count(rows, V, dc->num_sms);
+  void* parts = nullptr;
+  rc = scratch_reserve(dc, size_t(n) * rows * sizeof(Top1Part), &parts);
+  if (rc) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  launch_reduce_top1_parts(logits, rows, V, n, static_cast<Top1Part*>(parts), st);
+  launch_gate_transfer(static_cast<Top1Part*>(parts), n, nullptr, nullptr, conf, argmax, prev, persist, state, tokens,
+                       B, R, k, tau, K, unmask, accept, done, st);
+  CK(cudaGetLastError());
+  return CORA_OK;
+}
+
+extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32_t M, int32_t N, int32_t K,
+                            int32_t ldc, int32_t epilogue, const float* rope, int32_t seq, int32_t head_dim,
+                            int32_t rope_cols, void* stream) {
+  REQUIRE(A && B && C, "cora_op_gemm: NULL pointer");
+  REQUIRE(M >= 1 && N >= 128 && N % 128 == 0 && K >= 64 && K % 64 == 0, "cora_op_gemm: bad M/N/K");
+  REQUIRE(epilogue >= 0 && epilogue <= 3, "cora_op_gemm: bad epilogue");
+  REQUIRE(epilogue != CORA_EPI_SWIGLU || N % 256 == 0, "cora_op_gemm: SWIGLU needs N %% 256 == 0");
+  REQUIRE(aligned16(A) && aligned16(B) && aligned16(C), "cora_op_gemm: pointers must be 16-byte aligned");
+  const int out_cols = epilogue == CORA_EPI_SWIGLU ? N / 2 : N;
+  REQUIRE(ldc >= out_cols && ldc % 8 == 0, "cora_op_gemm: bad ldc");
+  if (epilogue == CORA_EPI_ROPE_BF16) {
+    REQUIRE(rope && seq >= 1 && (head_dim == 64 || head_dim == 128) && gemm_block_n(N, epilogue) % head_dim == 0,
+            "cora_op_gemm: bad RoPE arguments");
+  }
+  DeviceCtx* dc = nullptr;
+  int rc = device_ctx(&dc);
+  if (rc) return rc;
+  if ((rc = kernels_prepare())) return rc;
+  CUtensorMap ta, tb;
+  const int bn = gemm_block_n(N, epilogue);
+  if (!make_tmap_bf16_2d(&ta, A, M, K, size_t(K) * 2, 128, 64) || !make_tmap_bf16_2d(&tb, B, N, K, size_t(K) * 2, bn, 64))
+    return fail(CORA_ECUDA, "cora_op_gemm: tensor map encoding failed");
+  GemmEpilogue ep{C, ldc, epilogue, rope, seq, head_dim, rope_cols};
+  CK(launch_gemm(ta, tb, M, N, K, ep, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
+  return CORA_OK;
+}
+
+extern "C" int cora_op_attention(const uint16_t* qkv, uint16_t* out, int32_t B, int32_t S, int32_t Hq, int32_t Hkv,
+                                 int32_t hd, void* stream) {
+  REQUIRE(qkv && out, "cora_op_attention: NULL pointer");
+  REQUIRE(B >= 1 && S >= 1 && Hq >= 1 && Hkv >= 1 && Hq % Hkv == 0 && (hd == 64 || hd == 128),
+          "cora_op_attention: bad shape");
+  REQUIRE(aligned16(qkv) && aligned16(out), "cora_op_attention: pointers must be 16-byte aligned");
+  int rc = kernels_prepare();
+  if (rc) return rc;
+  launch_attention(qkv, out, B, S, Hq, Hkv, hd, static_cast<cudaStream_t>(stream));
+  CK(cudaGetLastError());
+  return CORA_OK;
+}
+
+extern "C" int cora_op_rmsnorm(const float* x, const uint16_t* w, uint16_t* out, int32_t M, int32_t d, float eps,
+                               void* stream) {
+  REQUIRE(x && out, "cora_op_rmsnorm: NULL pointer");
+  REQUIRE(M >= 1 && d >= 8 && d % 8 == 0, "cora_op_rmsnorm: bad shape");
+  REQUIRE(aligned16(x) && aligned16(out) && (!w || aligned16(w)), "cora_op_rmsnorm: pointers must be 16-byte aligned");
+  launch_rmsnorm(x, w, out, M, d, eps, static_cast<cudaStream_t>(stream));
+  CK(cudaGetLastError());
+  return CORA_OK;
+}
+
+extern "C" int cora_op_lm_head_top1(const uint16_t* x, const uint16_t* W, int32_t R, int32_t V, int32_t d, float* conf,
+                                    int32_t* argmax, void* stream) {
+  REQUIRE(x && W && conf && argmax, "cora_op_lm_head_top1: NULL pointer");
+  REQUIRE(R >= 1 && R <= 256 && V >= 1 && d >= 64 && d % 64 == 0, "cora_op_lm_head_top1: bad shape");
+  REQUIRE(aligned16(x) && aligned16(W), "cora_op_lm_head_top1: pointers must be 16-byte aligned");
+  DeviceCtx* dc = nullptr;
+  int rc = device_ctx(&dc);
+  if (rc) return rc;
+  if ((rc = kernels_prepare())) return rc;
+  CUtensorMap tw, tx;
+  if (!make_tmap_bf16_2d(&tw, W, V, d, size_t(d) * 2, 128, 64) ||
+      !make_tmap_bf16_2d(&tx, x, R, d, size_t(d) * 2, lm_head_npad(R), 64))
+    return fail(CORA_ECUDA, "cora_op_lm_head_top1: tensor map encoding failed");
+  const int n = lm_head_parts_count(V, dc->num_sms);
+  void* parts = nullptr;
+  rc = scratch_reserve(dc, size_t(n) * R * sizeof(Top1Part), &parts);
+  if (rc) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CK(launch_lm_head_top1(tw, tx, R, V, d, static_cast<Top1Part*>(parts), n, dc->err, st));
+  launch_combine_top1(static_cast<Top1Part*>(parts), n, R, conf, argmax, st);
+  CK(cudaGetLastError());
+  return CORA_OK;
+}
+
+extern "C" int cora_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_t start, float scale,
+                                      void* stream) {
+  REQUIRE(out && count >= 0 && start >= 0, "cora_synth_normal_bf16: bad argument");
+  launch_synth_normal_bf16(out, count, key, start, scale, static_cast<cudaStream_t>(stream));
+  CK(cudaGetLastError());
+  return CORA_OK;
+}
+
+extern "C" int cora_device_error(int32_t* code, int32_t clear) {
+  REQUIRE(code, "cora_device_error: NULL pointer");
+  DeviceCtx* dc = nullptr;
+  int rc = device_ctx(&dc);
+  if (rc) return rc;
+  CK(cudaDeviceSynchronize());
+  CK(cudaMemcpy(code, dc->err, sizeof(int), cudaMemcpyDeviceToHost));
+  if (clear) CK(cudaMemset(dc->err, 0, sizeof(int)));
+  return CORA_OK;
+}
