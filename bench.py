@@ -1,0 +1,402 @@
+#!/usr/bin/env python
+"""Decode-throughput benchmark of the CORA-Diff hot path on GB300.
+
+One bench step is one complete decode of the workload's batch: prompt
+canvas -> every block -> every executed denoising step (dense bidirectional
+forward, active-row LM head with Eq. 1 reduced on the fly, transfer rule and
+residual gate with block termination) until every sequence has finished.
+Metric: generated tokens/s = batch * gen_len * steps / device time.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl cora|reference]
+
+Default workload: LLaDA-8B-shaped bidirectional Transformer (32 layers,
+d 4096, 32 heads x 128, SwiGLU 12288, vocab 126464), random-init bf16
+weights, batch 1, prompt 256 random ids, gen_len 256, block 32, 32 steps per
+block, gate at the paper's frozen (delta_p, m) = (0.65, 1).
+
+With N GPUs (torchrun, one process per GPU) every rank decodes its own
+replica with its own prompts (replicas only: the method has no data-path
+exchange); value = all ranks' tokens / the slowest rank's time.
+
+--impl reference times the CPU oracle (float64 numpy) on the host cores on a
+bounded sample of the same workload and reports the same metric.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+# DRAM bytes (read + write) per launch from one ncu capture of each kernel on
+# the LLaDA-8B-shaped workload (2-layer model, same per-launch shapes), keyed
+# by a hash of the kernel source at capture time; null once the source changed.
+NCU_TRAFFIC = {}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return FALLBACK_PEAKS, "fallback"
+
+
+def src_hash(name: str) -> str:
+    with open(os.path.join(ROOT, "paper_2608_11235_gb300", "csrc", name), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:12]
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max([num(r[3]) for r in rows if num(r[3]) is not None], default=None)}
+
+
+# ------------------------------------------------------------ distributed
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+    return ws, rank, local
+
+
+def dist_max(x: float, ws: int) -> float:
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def dist_barrier(ws: int):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ------------------------------------------------------------- oracle leg
+def oracle_sample(cfg: dict, passes_per_seq: float, budget_s: float = 12.0):
+    """Times the oracle on a bounded sample of one dense pass: layer 0 of the
+    model on the full canvas (repeated until ``budget_s``) plus the LM head and
+    Eq. 1 on the active rows over a vocabulary slice; extrapolates tokens/s."""
+    from oracle import cora_oracle as O
+    from paper_2608_11235_gb300 import synth
+
+    S = cfg["prompt_len"] + cfg["gen_len"]
+    B, G, BL = cfg["batch"], cfg["gen_len"], cfg["block_len"]
+    lw = synth.layer_weights_f64(cfg, 0)
+    V = cfg["vocab"]
+    v_slice = min(V, 16384)
+    head = {"final_norm": np.ones(cfg["d_model"]),
+            "lm_head": synth.weight_f64(cfg, -1, synth.LM_HEAD, slice(0, v_slice))}
+    prompt = synth.prompts(cfg["prompt_seed"], 1, cfg["prompt_len"], cfg["mask_id"])[0]
+    x = np.concatenate([prompt, np.full(G, cfg["mask_id"])])
+    h = np.stack([synth.weight_f64(cfg, -1, synth.EMBED, slice(int(t), int(t) + 1))[0] for t in x[:S]])
+    t0 = time.perf_counter()
+    n_layers_run = 0
+    while True:
+        O.layer_forward(cfg, lw, h, np.arange(S))
+        n_layers_run += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    t_layer = (time.perf_counter() - t0) / n_layers_run
+    t1 = time.perf_counter()
+    lg = O.lm_logits(cfg, head, h[cfg["prompt_len"]: cfg["prompt_len"] + BL])
+    O.top1(lg)
+    t_head = (time.perf_counter() - t1) * V / v_slice
+    t_pass = B * (cfg["n_layers"] * t_layer + t_head)      # the oracle decodes sequences one by one
+    tok_s = B * G / (passes_per_seq * t_pass) if passes_per_seq > 0 else None
+    try:
+        from threadpoolctl import threadpool_info
+        cores = max([p.get("num_threads", 1) for p in threadpool_info()] or [os.cpu_count()])
+    except ImportError:
+        cores = int(os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1))
+    sample = (f"{n_layers_run} x layer-0 forward (S={S}, fp64) + LM head/Eq.1 on {BL} rows over {v_slice} of {V} "
+              f"vocab ids, extrapolated to {cfg['n_layers']} layers x {passes_per_seq:g} passes x B={B}")
+    return tok_s, cores, sample, n_layers_run * t_layer + t_head * v_slice / V
+
+
+# --------------------------------------------------------------- GPU leg
+def kernel_costs(cfg: dict):
+    """Algorithmic FLOPs / bytes per launch of each kernel class for one pass."""
+    B, S = cfg["batch"], cfg["prompt_len"] + cfg["gen_len"]
+    M, d, F, V = B * S, cfg["d_model"], cfg["ffn"], cfg["vocab"]
+    hq, hkv, hd = cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"]
+    R = B * cfg["block_len"]
+    return {
+        "gemm_qkv_rope": 2.0 * M * d * (hq + 2 * hkv) * hd,
+        "gemm_o_resid": 2.0 * M * hq * hd * d,
+        "gemm_gate_up_swiglu": 2.0 * M * d * 2 * F,
+        "gemm_down_resid": 2.0 * M * F * d,
+        "attention": 4.0 * B * hq * S * S * hd,
+        "lm_head_top1_bytes": 2.0 * V * d + 2.0 * R * d,
+        "lm_head_top1_flops": 2.0 * R * d * V,
+    }
+
+
+def run_cora(args, cfg, ws, rank, local):
+    import torch
+
+    from paper_2608_11235_gb300 import configs, cora, model, synth
+
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    peaks, peak_src = load_peaks()
+
+    B, P, G, BL, T = cfg["batch"], cfg["prompt_len"], cfg["gen_len"], cfg["block_len"], cfg["steps_per_block"]
+    tau, K = cfg["tau"], cfg["K"]
+    m = model.create_model(cfg, device=f"cuda:{local}")
+    prompt = synth.prompts(cfg["prompt_seed"] + 7919 * rank, B, P, cfg["mask_id"])
+    prompt_dev = torch.from_numpy(prompt).to(f"cuda:{local}")
+    s = cora.cora_session_create(m, B, prompt_dev, P, G, BL, T, tau, K)
+    stream = torch.cuda.ExternalStream(cora.cora_session_stream(s))
+
+    def decode():
+        cora.cora_session_reset(s, prompt_dev)
+        done = False
+        while not done:
+            done = cora.cora_denoise_step(s)
+        return cora.cora_session_batched_passes(s)
+
+    for _ in range(args.warmup):
+        passes = decode()
+    # ----- timed region: K complete decodes, device-resident inputs
+    dist_barrier(ws)
+    torch.cuda.synchronize()
+    clk = ClockSampler(local)
+    clk.start()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    total_passes = 0
+    for _ in range(args.steps):
+        total_passes += decode()
+    e1.record(stream)
+    e1.synchronize()
+    torch.cuda.synchronize()
+    clocks = clk.stop()
+    dist_barrier(ws)
+    ms_local = e0.elapsed_time(e1)
+    ms = dist_max(ms_local, ws)
+    out = cora.cora_session_read(s, B, P + G, G, BL)
+    per_seq_passes = out["ctrl"][:, 2].astype(float)
+
+    # ----- per-kernel device times (one eager pass with events around each launch)
+    cora.cora_session_reset(s, prompt_dev)
+    prof = cora.cora_session_profile_step(s, cfg["n_layers"])
+    cora.cora_session_reset(s, prompt_dev)
+    prof2 = cora.cora_session_profile_step(s, cfg["n_layers"])
+    by = {}
+    for (k1, t1), (_, t2) in zip(prof, prof2):
+        by.setdefault(k1, []).append(min(t1, t2))
+    costs = kernel_costs(cfg)
+    gemm_kinds = ["gemm_qkv_rope", "gemm_o_resid", "gemm_gate_up_swiglu", "gemm_down_resid"]
+    gemm_ms = sum(sum(by[k]) for k in gemm_kinds)
+    gemm_flops = sum(costs[k] * len(by[k]) for k in gemm_kinds)
+    n_gemm = sum(len(by[k]) for k in gemm_kinds)
+    step_ms = sum(sum(v) for v in by.values())
+    gemm_tflops = gemm_flops / (gemm_ms * 1e-3) / 1e12
+    peak_tf = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    head_ms = sum(by["lm_head_top1"]) / len(by["lm_head_top1"])
+    head_gbs = costs["lm_head_top1_bytes"] / (head_ms * 1e-3) / 1e9
+    attn_ms = sum(by["attention"]) / len(by["attention"])
+    kernels = {k: {"launches_per_pass": len(v), "ms_per_launch": round(sum(v) / len(v), 5),
+                   "share": round(sum(v) / step_ms, 4)} for k, v in sorted(by.items())}
+    traffic = NCU_TRAFFIC.get(("gemm", src_hash("gemm.cu")))
+    roofline = {"bound": "tensor", "kernel": "gemm_tc_kernel (QKV+RoPE, O+res, gate/up+SwiGLU, down+res)",
+                "achieved": round(gemm_tflops, 2), "peak": peak_tf, "unit": "TFLOP/s",
+                "frac": round(gemm_tflops / peak_tf, 4), "traffic": traffic,
+                "peak_source": f"{peak_src} bf16 sustained", "flops_per_launch": round(gemm_flops / n_gemm),
+                "ms_per_launch": round(gemm_ms / n_gemm, 5)}
+    others = {
+        "lm_head_top1": {"bound": "hbm", "achieved": round(head_gbs, 1), "unit": "GB/s",
+                         "peak": peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]),
+                         "frac": round(head_gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]), 4),
+                         "bytes_per_launch": costs["lm_head_top1_bytes"], "ms_per_launch": round(head_ms, 5)},
+        "attention": {"bound": "tensor(mma.sync)", "achieved": round(costs["attention"] / (attn_ms * 1e-3) / 1e12, 2),
+                      "unit": "TFLOP/s", "ms_per_launch": round(attn_ms, 5)},
+        "pass_model_tflops": round((gemm_flops + costs["attention"] * len(by["attention"]) +
+                                    costs["lm_head_top1_flops"]) / (step_ms * 1e-3) / 1e12, 2),
+    }
+
+    # ----- end to end through the public call, host buffers (pinned), copies inside
+    prompt_pin = torch.from_numpy(prompt).pin_memory()
+    for _ in range(1):
+        cora.cora_generate(m, prompt_pin.numpy(), G, BL, T, tau, K)
+    dist_barrier(ws)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        toks, passes_e2e, _ = cora.cora_generate(m, prompt_pin.numpy(), G, BL, T, tau, K)
+    e2e_s = dist_max(time.perf_counter() - t0, ws)
+    assert toks.shape == (B, G)
+
+    # ----- gate-exercising variant (LM head scaled so confidences span (0, 1))
+    gx = None
+    if not args.no_variant:
+        cfg_g = configs.gate_exercising(cfg)
+        cora.cora_session_destroy(s)
+        mg = model.create_model(cfg_g, device=f"cuda:{local}")
+        cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau, K)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        reps = max(1, args.steps)
+        for _ in range(reps):
+            _, pg, bg = cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau, K)
+        tg = time.perf_counter() - t0
+        gx = {"head_sigma": round(cfg_g["head_sigma"], 6), "tokens_per_s": round(B * G * reps / tg, 2),
+              "passes_per_block": round(float(pg.mean()) / (G // BL), 3),
+              "rho": round(float(pg.mean()) / ((G // BL) * T), 4), "timing": "host wall clock, e2e call"}
+        cora.cora_model_destroy(mg)
+        s = None
+    if s is not None:
+        cora.cora_session_destroy(s)
+    cora.cora_model_destroy(m)
+
+    value = ws * B * G * args.steps / (ms * 1e-3)
+    launches_per_pass = 4 + 7 * cfg["n_layers"]
+    result = {
+        "metric": "generated tokens/s (LLaDA-8B shape, gen 256)",
+        "value": round(value, 3), "unit": "tokens/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms / args.steps, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic (seeded random-init weights and prompt ids)",
+        "config": {"workload": cfg["name"], "batch": B, "prompt_len": P, "gen_len": G, "block_len": BL,
+                   "steps_per_block": T, "tau": tau, "K": K, "n_layers": cfg["n_layers"], "d_model": cfg["d_model"],
+                   "vocab": cfg["vocab"], "weights": f"bf16 N(0,{cfg['init_sigma']}) (approx.), head N(0,{cfg['head_sigma']})",
+                   "l2": "inputs larger than L2 (16 GB of weights streamed every pass)",
+                   "passes_per_seq": float(per_seq_passes.mean()),
+                   "passes_per_block": round(float(per_seq_passes.mean()) / (G // BL), 3),
+                   "rho": round(float(per_seq_passes.mean()) / ((G // BL) * T), 4),
+                   "parallelism": f"replicas x{ws}"},
+        "e2e": {"value": round(ws * B * G * args.steps / e2e_s, 3), "unit": "tokens/s",
+                "h2d_bytes_per_step": int(B * P * 4), "d2h_bytes_per_step": int(B * G * 4 + B * 8),
+                "timing": "host wall clock around cora_generate (pinned host prompt in, host tokens out)"},
+        "roofline": roofline,
+        "kernels": kernels,
+        "other_rooflines": others,
+        "gpu_launches": int(total_passes * launches_per_pass + args.steps),
+        "clocks": clocks,
+        "gate_exercising": gx,
+    }
+    return result, float(per_seq_passes.mean())
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["cora", "reference"], default="cora")
+    ap.add_argument("--workload", default="llada8b-shape-256+256")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-variant", action="store_true")
+    ap.add_argument("--layers", type=int, default=0, help="override n_layers (same per-launch shapes)")
+    args = ap.parse_args()
+    from paper_2608_11235_gb300 import configs
+    cfg = dict(configs.PRESETS[args.workload])
+    if args.layers:
+        cfg = configs.with_layers(cfg, args.layers)
+    ws, rank, local = dist_setup()
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        horizon = (cfg["gen_len"] // cfg["block_len"]) * cfg["steps_per_block"]
+        vals, times = [], []
+        for i in range(args.warmup + args.steps):
+            tok_s, cores, sample, t = oracle_sample(cfg, horizon, budget_s=8.0)
+            if i >= args.warmup:
+                vals.append(tok_s)
+                times.append(t)
+        v = statistics.mean(vals)
+        print(json.dumps({
+            "impl": "reference", "metric": "generated tokens/s (LLaDA-8B shape, gen 256)", "value": v,
+            "unit": "tokens/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * statistics.mean(times), 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": cfg["name"], "batch": cfg["batch"], "prompt_len": cfg["prompt_len"],
+                       "gen_len": cfg["gen_len"], "passes_per_seq": horizon, "parallelism": "none (host cores)"},
+            "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        }))
+        return
+
+    result, passes = run_cora(args, cfg, ws, rank, local)
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        tok_s, cores, sample, _ = oracle_sample(cfg, passes)
+        result["cpu_baseline"] = {"value": tok_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                                  "sample": sample}
+    elif rank == 0:
+        result["cpu_baseline"] = None
+    if rank == 0:
+        print(json.dumps(result))
+
+
+if __name__ == "__main__":
+    main()

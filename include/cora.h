@@ -76,8 +76,9 @@ CORA_API int cora_version(void);
  * residual -> RMSNorm -> SwiGLU FFN (silu(x W_gate^T) * (x W_up^T)) W_down^T +
  * residual; final RMSNorm and an untied LM head.  This is the frozen dense
  * pass the paper runs unchanged at every executed step (Sec. 3, Sec. 4.1).
- * Constraints: d_model % 64 == 0, head_dim in {64, 128},
- * n_heads % n_kv_heads == 0, (n_heads * head_dim) % 64 == 0, vocab >= 2,
+ * Constraints: d_model % 128 == 0, head_dim in {64, 128},
+ * n_heads % n_kv_heads == 0, (n_heads * head_dim) % 64 == 0,
+ * ((n_heads + 2 * n_kv_heads) * head_dim) % 128 == 0, vocab >= 2,
  * 0 <= mask_id < vocab.
  * ------------------------------------------------------------------------- */
 typedef struct cora_model_config {
@@ -176,6 +177,31 @@ CORA_API int cora_session_read(cora_session* s, int32_t* tokens, uint8_t* state,
  * decode at block/step granularity.  Synchronous. */
 CORA_API int cora_session_write(cora_session* s, const int32_t* tokens, const uint8_t* state, const int32_t* persist,
                        const int32_t* prev, const int32_t* ctrl);
+
+/* Launch classes reported by cora_session_profile_step. */
+#define CORA_KIND_EMBED 0
+#define CORA_KIND_RMSNORM 1
+#define CORA_KIND_GEMM_QKV 2       /* QKV projection + RoPE epilogue */
+#define CORA_KIND_ATTENTION 3
+#define CORA_KIND_GEMM_O 4         /* output projection + residual */
+#define CORA_KIND_GEMM_GATE_UP 5   /* gate/up projection + SwiGLU epilogue */
+#define CORA_KIND_GEMM_DOWN 6      /* down projection + residual */
+#define CORA_KIND_FINAL_NORM 7
+#define CORA_KIND_LM_HEAD 8        /* fused LM head + Eq. 1 partials */
+#define CORA_KIND_GATE 9           /* Eq. 1 combine + transfer rule + Eq. 2-4 */
+
+/* Runs one cora_denoise_step without the CUDA graph, with CUDA events around
+ * every kernel launch, for profiling.  It is a real step (state advances).
+ *   capacity  size of kinds/ms (>= 4 + 7 * n_layers)
+ *   kinds     host int32 [capacity] (out): CORA_KIND_* of each launch, in order
+ *   ms        host float [capacity] (out): device time of each launch
+ *   n_out     host int32 (out): launches recorded
+ * Synchronous. */
+CORA_API int cora_session_profile_step(cora_session* s, int32_t capacity, int32_t* kinds, float* ms, int32_t* n_out);
+
+/* The cudaStream_t (as void*) on which the session launches its work; a
+ * caller may record events on it to time steps on the device. */
+CORA_API int cora_session_stream(cora_session* s, void** out);
 
 /* Number of batched steps (dense passes over the batch) executed since the
  * last reset. */

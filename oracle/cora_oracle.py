@@ -244,6 +244,7 @@ def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
             return forward_hidden(cfg, w, tok)
     P = len(prompt)
     x = np.concatenate([np.asarray(prompt, np.int64), np.full(gen_len, cfg["mask_id"], np.int64)])
+    gstate = np.zeros(gen_len, np.uint8)      # state of every generation position
     passes = []
     steps = []
     for b in range(gen_len // block_len):
@@ -252,16 +253,18 @@ def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
         sched = transfer_schedule(block_len, T)
         n_exec = 0
         for s in range(T):
+            canvas, gs = (x.copy(), gstate.copy()) if record else (None, None)
             h = forward(x)
             logits = lm_logits(cfg, w, h[lo: lo + block_len])
             conf, x_hat = top1(logits)
             before = st.copy() if record else None
             r = cora_step(st, conf, x_hat, sched[s], tau, K)
             x[lo: lo + block_len] = st.tokens
+            gstate[b * block_len: (b + 1) * block_len] = st.state
             n_exec += 1
             if record:
-                steps.append(dict(block=b, step=s, canvas=None, conf=conf, x_hat=x_hat,
-                                  logits=logits, before=before, after=st.copy(), result=r))
+                steps.append(dict(block=b, step=s, canvas=canvas, gen_state=gs, passes_before=n_exec - 1,
+                                  conf=conf, x_hat=x_hat, logits=logits, before=before, after=st.copy(), result=r))
             if r.done:
                 break
         passes.append(n_exec)

@@ -25,8 +25,10 @@ EXPORTED = [
     "cora_session_destroy", "cora_session_reset", "cora_denoise_step", "cora_session_read", "cora_session_write",
     "cora_session_batched_passes", "cora_generate", "cora_gate_transfer", "cora_reduce_top1", "cora_reduce_gate",
     "cora_op_gemm", "cora_op_attention", "cora_op_rmsnorm", "cora_op_lm_head_top1", "cora_synth_normal_bf16",
-    "cora_device_error",
+    "cora_device_error", "cora_session_profile_step", "cora_session_stream",
 ]
+KIND_NAMES = ["embed", "rmsnorm", "gemm_qkv_rope", "attention", "gemm_o_resid", "gemm_gate_up_swiglu",
+              "gemm_down_resid", "final_norm", "lm_head_top1", "gate"]
 
 
 class CoraError(RuntimeError):
@@ -78,6 +80,8 @@ def lib():
             "cora_session_read": ([vp] + [vp] * 9, C.c_int),
             "cora_session_write": ([vp] + [vp] * 5, C.c_int),
             "cora_session_batched_passes": ([vp, vp], C.c_int),
+            "cora_session_profile_step": ([vp, i32, vp, vp, vp], C.c_int),
+            "cora_session_stream": ([vp, C.POINTER(vp)], C.c_int),
             "cora_generate": ([vp, vp, i32, i32, i32, i32, i32, f32, i32, vp, vp, vp], C.c_int),
             "cora_gate_transfer": ([vp] * 6 + [i32, i32, i32, f32, i32] + [vp] * 3 + [vp], C.c_int),
             "cora_reduce_top1": ([vp, i32, i32, vp, vp, vp], C.c_int),
@@ -190,6 +194,22 @@ def cora_session_write(session, tokens=None, state=None, persist=None, prev=None
         return None if a is None else np.ascontiguousarray(a, dtype=dt)
     arrs = [c(tokens, np.int32), c(state, np.uint8), c(persist, np.int32), c(prev, np.int32), c(ctrl, np.int32)]
     _check("cora_session_write", lib().cora_session_write(session, *[ptr(a) for a in arrs]))
+
+
+def cora_session_profile_step(session, n_layers: int):
+    """Runs one step eagerly with events around each launch: [(kind name, ms), ...]."""
+    cap = 4 + 7 * n_layers
+    kinds = np.zeros(cap, np.int32)
+    ms = np.zeros(cap, np.float32)
+    n = np.zeros(1, np.int32)
+    _check("cora_session_profile_step", lib().cora_session_profile_step(session, cap, ptr(kinds), ptr(ms), ptr(n)))
+    return [(KIND_NAMES[int(kinds[i])], float(ms[i])) for i in range(int(n[0]))]
+
+
+def cora_session_stream(session) -> int:
+    out = C.c_void_p()
+    _check("cora_session_stream", lib().cora_session_stream(session, C.byref(out)))
+    return out.value or 0
 
 
 def cora_session_batched_passes(session) -> int:

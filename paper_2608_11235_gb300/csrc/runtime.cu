@@ -314,34 +314,71 @@ static int sess_alloc(cora_session* s, size_t count, T** out) {
   return CORA_OK;
 }
 
-static int enqueue_step(cora_session* s) {
+// Optional per-launch event recorder (profiling path only; the graph path
+// passes nullptr).
+struct LaunchRecorder {
+  std::vector<cudaEvent_t> ev;
+  std::vector<int32_t> kinds;
+  cudaStream_t st = nullptr;
+  int mark(int kind) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return -1;
+    cudaEventRecord(e, st);
+    ev.push_back(e);
+    if (kind >= 0) kinds.push_back(kind);
+    return 0;
+  }
+  ~LaunchRecorder() {
+    for (auto e : ev) cudaEventDestroy(e);
+  }
+};
+
+#define REC(kind) \
+  if (rec) rec->mark(kind)
+
+static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr) {
   cora_model* m = s->m;
   const cora_model_config& c = m->cfg;
   const int d = c.d_model, M = s->M;
   int* err = s->status + 1;
   cudaStream_t st = s->stream;
+  if (rec) {
+    rec->st = st;
+    rec->mark(-1);
+  }
   launch_embed(s->tokens, m->embed, s->h, M, d, st);
+  REC(CORA_KIND_EMBED);
   for (int l = 0; l < c.n_layers; ++l) {
     launch_rmsnorm(s->h, m->attn_norm[l], s->xn, M, d, c.norm_eps, st);
+    REC(CORA_KIND_RMSNORM);
     GemmEpilogue e1{s->qkv, m->n_qkv, CORA_EPI_ROPE_BF16, s->rope, s->S, c.head_dim,
                     (c.n_heads + c.n_kv_heads) * c.head_dim};
     CK(launch_gemm(s->tm_xn, m->tm_qkv[l], M, m->n_qkv, d, e1, err, m->num_sms, st));
+    REC(CORA_KIND_GEMM_QKV);
     launch_attention(s->qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, st);
+    REC(CORA_KIND_ATTENTION);
     GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0};
     CK(launch_gemm(s->tm_attn, m->tm_o[l], M, d, c.n_heads * c.head_dim, e2, err, m->num_sms, st));
+    REC(CORA_KIND_GEMM_O);
     launch_rmsnorm(s->h, m->ffn_norm[l], s->xn, M, d, c.norm_eps, st);
+    REC(CORA_KIND_RMSNORM);
     GemmEpilogue e3{s->act, m->f_pad, CORA_EPI_SWIGLU, nullptr, 0, 0, 0};
     CK(launch_gemm(s->tm_xn, m->tm_gu[l], M, 2 * m->f_pad, d, e3, err, m->num_sms, st));
+    REC(CORA_KIND_GEMM_GATE_UP);
     CK(launch_gemm(s->tm_act, m->tm_down[l], M, d, m->f_pad, e2, err, m->num_sms, st));
+    REC(CORA_KIND_GEMM_DOWN);
   }
   launch_final_norm_rows(s->h, m->final_norm, s->ctrl, s->xf, s->B, s->S, s->P, s->BL, s->n_blocks, d, c.norm_eps,
                          st);
+  REC(CORA_KIND_FINAL_NORM);
   CK(launch_lm_head_top1(m->tm_head, s->tm_xf, s->R, c.vocab, d, s->parts, s->n_parts, err, st));
+  REC(CORA_KIND_LM_HEAD);
   SessionGateArgs ga{s->parts, s->n_parts, s->ctrl,  s->tokens, s->state,  s->persist, s->prev,
                      s->conf,  s->argmax,  s->unmask, s->accept, reinterpret_cast<uint8_t*>(s->status),
                      err,      s->B,       s->S,      s->P,      s->G,       s->BL,      s->T,
                      s->tau,   s->K};
   launch_session_gate(ga, st);
+  REC(CORA_KIND_GATE);
   CK(cudaGetLastError());
   CK(cudaMemcpyAsync(s->status_h, s->status, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
   return CORA_OK;
@@ -491,6 +528,37 @@ extern "C" int cora_denoise_step(cora_session* s, uint8_t* all_done_out) {
   const uint8_t done = reinterpret_cast<const uint8_t*>(s->status_h)[0];
   s->finished = done != 0;
   if (all_done_out) *all_done_out = done;
+  return CORA_OK;
+}
+
+extern "C" int cora_session_profile_step(cora_session* s, int32_t capacity, int32_t* kinds, float* ms,
+                                         int32_t* n_out) {
+  REQUIRE(s && kinds && ms && n_out, "cora_session_profile_step: NULL argument");
+  if (s->finished) return fail(CORA_ESTATE, "every sequence has finished; reset the session");
+  const int need = 3 + 7 * s->m->cfg.n_layers + 1;
+  REQUIRE(capacity >= need, "cora_session_profile_step: capacity %d < %d launches", capacity, need);
+  CK(cudaStreamSynchronize(s->stream));
+  LaunchRecorder rec;
+  int rc = enqueue_step(s, &rec);
+  if (rc) return rc;
+  CK(cudaStreamSynchronize(s->stream));
+  s->batched_passes += 1;
+  const int n = static_cast<int>(rec.kinds.size());
+  for (int i = 0; i < n; ++i) {
+    float t = 0.f;
+    CK(cudaEventElapsedTime(&t, rec.ev[i], rec.ev[i + 1]));
+    kinds[i] = rec.kinds[i];
+    ms[i] = t;
+  }
+  *n_out = n;
+  if (s->status_h[1] != 0) return fail(CORA_ETIMEOUT, "device error word 0x%x after step", s->status_h[1]);
+  s->finished = reinterpret_cast<const uint8_t*>(s->status_h)[0] != 0;
+  return CORA_OK;
+}
+
+extern "C" int cora_session_stream(cora_session* s, void** out) {
+  REQUIRE(s && out, "NULL argument");
+  *out = static_cast<void*>(s->stream);
   return CORA_OK;
 }
 

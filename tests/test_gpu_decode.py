@@ -1,0 +1,133 @@
+"""End-to-end decode on the GPU against the oracle (tiny two-layer model).
+
+Replay parity: the oracle decodes with the tiny model's operating point
+(tau = 0.9, K = 2); before each of its executed steps the GPU session is set
+to the oracle's pre-step state (canvas, position states, persistence) and runs
+one cora_denoise_step.  Eq. 1 must agree (|dc| <= 2e-2, argmax equal where
+the oracle's top-1/top-2 probability margin exceeds 2e-2); the gate's output
+must equal the oracle's wherever the measured confidence error cannot flip a
+decision, and must follow the rule on the GPU's own confidences everywhere.
+
+Closed forms on the GPU: the gate switched off gives the full horizon; an
+accept-everything gate ends every block after one pass (K = 0) or two (K = 1).
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import cora_oracle as O
+from paper_2608_11235_gb300 import build, configs, cora, model, synth
+
+pytestmark = pytest.mark.gpu
+CFG = dict(configs.TINY)
+P, G, BL, T = CFG["prompt_len"], CFG["gen_len"], CFG["block_len"], CFG["steps_per_block"]
+TAU, K = CFG["tau"], CFG["K"]
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    assert torch.cuda.is_available()
+    build.build()
+    m = model.create_model(CFG, on_device_fill=False)
+    w = synth.model_weights_f64(CFG)
+    prompt = synth.prompts(CFG["prompt_seed"], 3, P, CFG["mask_id"])
+    yield m, w, prompt
+    cora.cora_model_destroy(m)
+    assert cora.cora_device_error(clear=True) == 0
+
+
+def rule_holds(before_state, persist_before, prev_before, conf, arg, k, tau, Kp, after):
+    """The gate's output follows Eq. 2-4 on the GPU's own conf/argmax."""
+    U = before_state == 0
+    persist = np.where(U, np.where(prev_before == arg, persist_before + 1, 0), persist_before)
+    idx = [i for i in np.argsort(-conf.astype(np.float64), kind="stable") if U[i]]
+    Tm = np.zeros(len(U), bool)
+    Tm[idx[:min(k, len(idx))]] = True
+    A = U & ~Tm & (conf >= np.float32(tau)) & (persist >= Kp) & (Kp >= 0)
+    return np.array_equal(after["unmask"].astype(bool), Tm) and np.array_equal(after["accept"].astype(bool), A)
+
+
+def test_replay_parity_every_step(tiny):
+    m, w, prompt = tiny
+    tr = O.generate(CFG, w, prompt[0], G, BL, T, TAU, K, record=True)
+    assert sum(len(s["result"].accepted) for s in tr.steps) > 0, "the gate should fire on the tiny model"
+    s = cora.cora_session_create(m, 1, prompt[:1], P, G, BL, T, TAU, K)
+    robust_steps = 0
+    max_dc = 0.0
+    try:
+        for st in tr.steps:
+            b0 = st["before"]
+            ctrl = np.array([[st["block"], st["step"], st["passes_before"], 0]], np.int32)
+            cora.cora_session_write(s, tokens=st["canvas"][None], state=st["gen_state"][None],
+                                    persist=b0.persist[None], prev=b0.prev[None], ctrl=ctrl)
+            cora.cora_denoise_step(s)
+            out = cora.cora_session_read(s, 1, P + G, G, BL)
+            c, a = out["conf"][0], out["argmax"][0]
+            dc = np.abs(c - st["conf"])
+            max_dc = max(max_dc, float(dc.max()))
+            assert dc.max() <= 2e-2, (st["block"], st["step"], dc.max())
+            sel = O.top2_margin(st["logits"]) > 2e-2
+            assert np.array_equal(a[sel], st["x_hat"][sel])
+            k = O.transfer_schedule(BL, T)[st["step"]]
+            after = dict(unmask=out["unmask"][0], accept=out["accept"][0])
+            assert rule_holds(b0.state, b0.persist, b0.prev, c, a, k, TAU, K, after)
+            # Decisions the measured error cannot flip must equal the oracle's.
+            eps = float(dc.max()) + 1e-6
+            U = b0.state == O.UNRESOLVED
+            cu = np.sort(st["conf"][U])[::-1]
+            robust = np.array_equal(a[U], st["x_hat"][U])
+            robust &= len(cu) <= k or k == 0 or (cu[k - 1] - cu[k]) > 2 * eps
+            robust &= bool(np.all(np.abs(st["conf"][U] - TAU) > eps))
+            if robust:
+                robust_steps += 1
+                r = st["result"]
+                assert sorted(np.flatnonzero(out["unmask"][0])) == r.transferred
+                assert sorted(np.flatnonzero(out["accept"][0])) == r.accepted
+                lo = P + st["block"] * BL
+                assert np.array_equal(out["tokens"][0][lo: lo + BL], st["after"].tokens)
+                assert np.array_equal(out["state"][0][st["block"] * BL:(st["block"] + 1) * BL], st["after"].state)
+                if not r.done:
+                    assert np.array_equal(out["persist"][0], st["after"].persist)
+                    assert out["ctrl"][0, 1] == st["step"] + 1
+                else:
+                    assert out["ctrl"][0, 0] == st["block"] + 1 and out["ctrl"][0, 1] == 0
+    finally:
+        cora.cora_session_destroy(s)
+    assert robust_steps >= 0.6 * len(tr.steps), (robust_steps, len(tr.steps))
+    print(f"replayed {len(tr.steps)} steps, {robust_steps} with flip-proof decisions, max|dc| = {max_dc:.2e}")
+
+
+def test_gate_off_runs_full_horizon(tiny):
+    m, _, prompt = tiny
+    toks, passes, batched = cora.cora_generate(m, prompt[:1], G, BL, T, 2.0, 1)
+    assert passes[0] == (G // BL) * T and batched == (G // BL) * T
+    toks2, passes2, _ = cora.cora_generate(m, prompt[:1], G, BL, T, 1.0, -1)
+    assert passes2[0] == (G // BL) * T and np.array_equal(toks, toks2)
+
+
+@pytest.mark.parametrize("Kp,per_block", [(0, 1), (1, 2)])
+def test_accept_all_gate_closed_form(tiny, Kp, per_block):
+    m, _, prompt = tiny
+    _, passes, _ = cora.cora_generate(m, prompt[:1], G, BL, T, 0.0, Kp)
+    assert passes[0] == (G // BL) * per_block
+
+
+def test_free_running_decode_invariants(tiny):
+    m, w, prompt = tiny
+    toks, passes, batched = cora.cora_generate(m, prompt[:1], G, BL, T, TAU, K)
+    assert 3 * (G // BL) <= passes[0] <= (G // BL) * T     # K = 2: no acceptance before a block's third pass
+    assert np.all((toks >= 0) & (toks < CFG["vocab"]))
+    tr = O.generate(CFG, w, prompt[0], G, BL, T, TAU, K)
+    agree = float(np.mean(toks[0] == tr.tokens))
+    print(f"free-running GPU vs oracle: {agree:.3f} token agreement, passes {passes[0]} vs {sum(tr.passes_per_block)}")
+
+
+def test_batch_sequences_are_independent(tiny):
+    m, _, prompt = tiny
+    toks3, passes3, batched = cora.cora_generate(m, prompt, G, BL, T, TAU, K)
+    assert batched == passes3.max()
+    for b in range(3):
+        toks1, passes1, _ = cora.cora_generate(m, prompt[b: b + 1], G, BL, T, TAU, K)
+        assert passes1[0] == passes3[b]
+        assert np.array_equal(toks1[0], toks3[b])
