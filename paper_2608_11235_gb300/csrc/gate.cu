@@ -94,13 +94,28 @@ __device__ __forceinline__ Top1 combine_parts(const Top1Part* __restrict__ parts
   return st;
 }
 
+// One warp combines the partials of one row: lane l merges partials l, l+32,
+// ... in order, then the lanes merge in a fixed butterfly (deterministic).
+__device__ __forceinline__ Top1 warp_combine_parts(const Top1Part* __restrict__ parts, int n_parts, int rows,
+                                                   int row) {
+  const int lane = threadIdx.x & 31;
+  Top1 st = top1_empty();
+  for (int q = lane; q < n_parts; q += 32) {
+    const Top1Part pp = parts[static_cast<int64_t>(q) * rows + row];
+    st = top1_merge(st, Top1{pp.m, pp.s, pp.idx});
+  }
+  return warp_merge(st);
+}
+
 __global__ void combine_top1_kernel(const Top1Part* __restrict__ parts, int n_parts, int rows,
                                     float* __restrict__ conf, int32_t* __restrict__ argmax) {
-  const int row = blockIdx.x * blockDim.x + threadIdx.x;
-  if (row >= rows) return;
-  const Top1 st = combine_parts(parts, n_parts, rows, row);
-  conf[row] = 1.f / st.s;  // max_v softmax = exp(m - m) / sum exp(l - m)
-  argmax[row] = st.idx;
+  const int row = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (row >= rows) return;  // warp-uniform
+  const Top1 st = warp_combine_parts(parts, n_parts, rows, row);
+  if ((threadIdx.x & 31) == 0) {
+    conf[row] = 1.f / st.s;  // max_v softmax = exp(m - m) / sum exp(l - m)
+    argmax[row] = st.idx;
+  }
 }
 
 // ------------------------------------------------------------ Eq. 2-4 (K10)
@@ -196,6 +211,17 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
   const int lane = threadIdx.x & 31;
   const int nw = blockDim.x >> 5;
   const int n_blocks = a.G / a.BL;
+  const int R = a.B * a.BL;
+  // Eq. 1: every warp combines whole rows' partials (rows of finished
+  // sequences included; they are ignored below).
+  for (int r = threadIdx.x >> 5; r < R; r += nw) {
+    const Top1 st = warp_combine_parts(a.parts, a.n_parts, R, r);
+    if (lane == 0) {
+      a.conf[r] = 1.f / st.s;
+      a.argmax[r] = st.idx;
+    }
+  }
+  __syncthreads();
   for (int b = threadIdx.x >> 5; b < a.B; b += nw) {
     int32_t* ctrl = a.ctrl + b * 4;
     if (ctrl[3]) continue;  // finished: nothing to do (warp-uniform)
@@ -206,11 +232,8 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
     const int64_t gpos = static_cast<int64_t>(b) * a.G + static_cast<int64_t>(blk) * a.BL + lane;
     GateLane g{};
     if (valid) {
-      const Top1 st = combine_parts(a.parts, a.n_parts, a.B * a.BL, r);
-      g.c = 1.f / st.s;
-      g.xhat = st.idx;
-      a.conf[r] = g.c;
-      a.argmax[r] = g.xhat;
+      g.c = a.conf[r];
+      g.xhat = a.argmax[r];
       g.prev = a.prev[r];
       g.persist = a.persist[r];
       g.state = a.state[gpos];
@@ -273,7 +296,7 @@ void launch_reduce_top1_parts(const uint16_t* logits, int rows, int V, int n_chu
 
 void launch_combine_top1(const Top1Part* parts, int n_parts, int rows, float* conf, int32_t* argmax,
                          cudaStream_t st) {
-  combine_top1_kernel<<<(rows + 127) / 128, 128, 0, st>>>(parts, n_parts, rows, conf, argmax);
+  combine_top1_kernel<<<(rows + 7) / 8, 256, 0, st>>>(parts, n_parts, rows, conf, argmax);
 }
 
 void launch_gate_transfer(const Top1Part* parts, int n_parts, const float* conf_in, const int32_t* argmax_in,
@@ -287,6 +310,7 @@ void launch_gate_transfer(const Top1Part* parts, int n_parts, const float* conf_
 }
 
 void launch_session_gate(const SessionGateArgs& a, cudaStream_t st) {
-  int warps = a.B < 32 ? a.B : 32;
+  const int R = a.B * a.BL;
+  const int warps = R < 32 ? R : 32;
   session_gate_kernel<<<1, 32 * warps, 0, st>>>(a);
 }

@@ -94,7 +94,7 @@ def test_replay_parity_every_step(tiny):
                     assert out["ctrl"][0, 0] == st["block"] + 1 and out["ctrl"][0, 1] == 0
     finally:
         cora.cora_session_destroy(s)
-    assert robust_steps >= 0.6 * len(tr.steps), (robust_steps, len(tr.steps))
+    assert robust_steps >= 0.5 * len(tr.steps), (robust_steps, len(tr.steps))
     print(f"replayed {len(tr.steps)} steps, {robust_steps} with flip-proof decisions, max|dc| = {max_dc:.2e}")
 
 
