@@ -21,6 +21,7 @@
 #define CORA_DERR_TMA_WAIT 0x101
 #define CORA_DERR_MMA_WAIT 0x102
 #define CORA_DERR_EPI_WAIT 0x103
+#define CORA_DERR_SPLIT_WAIT 0x104
 #define CORA_DERR_GATE 0x201
 
 namespace cora {

@@ -68,13 +68,21 @@ struct GemmEpilogue {
   int rope_cols;
 };
 
+// Stream-K workspace: one fp32 partial slot of 128 x 256 per CTA plus one
+// flag per CTA (zero between launches).
+struct GemmWorkspace {
+  float* partial;
+  int* flags;
+};
+size_t gemm_workspace_bytes(int num_sms);
+
 // Tensor-map encoder (driver entry point fetched at runtime).
 bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
                        uint32_t box_rows, uint32_t box_cols);
 
 int gemm_block_n(int N, int mode);
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K,
-                        const GemmEpilogue& ep, int* err, int num_sms, cudaStream_t st);
+                        const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st);
 
 // Fused LM head + Eq. 1 partials: x [R, d] (tensor map box rows = n_pad),
 // W [V, d].  Writes parts [grid][R]; returns the number of parts used.

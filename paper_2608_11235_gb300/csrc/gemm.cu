@@ -2,7 +2,7 @@
 // backbone's projections: acc[M, N] = A[M, K] * B[N, K]^T, fp32 accumulation
 // in TMEM, operands staged in shared memory by TMA with 128-byte swizzling.
 //
-// Persistent kernel, one CTA per SM, 6 warps:
+// Persistent stream-K kernel, one CTA per SM, 6 warps:
 //   warp 0      TMA producer (one elected lane): A and B K-slices into a ring
 //               of STAGES shared-memory buffers (full/empty mbarriers);
 //   warp 1      TMEM allocator and MMA issuer (one lane): 128 x BN x 16
@@ -10,9 +10,22 @@
 //   warps 2..5  epilogue: tcgen05.ld of the 128 x BN accumulator (warp w
 //               reads TMEM lanes 32*(w%4) .. +31, one output row per thread),
 //               fused epilogue, global stores.
-// Two TMEM accumulators (2 * BN columns) let the epilogue of tile i overlap
-// the MMAs of tile i+1.  Tiles are visited M-fastest so the CTAs working at
-// the same time share the weight tile (B) through L2.
+//
+// Work split (stream-K): the (tile, k-block) iterations of the whole GEMM
+// are divided evenly among the CTAs, so every SM gets the same number of
+// MMAs whatever the tile count.  A CTA's range is contiguous; only its first
+// and last tile can be partial.  A tile split across CTAs is finished by the
+// CTA that holds its k-block 0 (which reaches it at the END of its range);
+// every other contributor writes its fp32 partial accumulator to its own
+// workspace slot at the START of its range and raises a flag.  The finishing
+// CTA adds the partials in increasing CTA order (deterministic), then runs the
+// epilogue.  All CTAs are co-resident (grid <= SMs, one CTA per SM), waits are
+// bounded, and the finishing CTA clears the flags it consumed.
+//
+// Tiles are ordered M-slowest, so at any moment the CTAs working on the same
+// weight tile (B) for different row blocks run concurrently and share it
+// through L2.  Two TMEM accumulators (2 * BN columns) let the epilogue of one
+// segment overlap the MMAs of the next.
 #include <math.h>
 
 #include "cora_device.cuh"
@@ -34,6 +47,26 @@ struct GemmCfg {
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 };
 
+// Contiguous, even split of W iterations over G CTAs.
+__device__ __forceinline__ int sk_start(int c, int G, int W) {
+  return static_cast<int>((static_cast<long long>(c) * W) / G);
+}
+
+// Walks a CTA's iteration range as segments (tile, kb0, kb1).
+struct SegIter {
+  int it, it_end, kb_per_tile;
+  __device__ SegIter(int c, int G, int W, int KB) : it(sk_start(c, G, W)), it_end(sk_start(c + 1, G, W)),
+                                                     kb_per_tile(KB) {}
+  __device__ bool next(int& t, int& kb0, int& kb1) {
+    if (it >= it_end) return false;
+    t = it / kb_per_tile;
+    kb0 = it - t * kb_per_tile;
+    kb1 = min(kb_per_tile, kb0 + (it_end - it));
+    it += kb1 - kb0;
+    return true;
+  }
+};
+
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + __expf(-x)); }
 
 __device__ __forceinline__ void store_bf16x16(uint16_t* dst, const float (&v)[16]) {
@@ -50,16 +83,48 @@ __device__ __forceinline__ void store_bf16x16(uint16_t* dst, const float (&v)[16
   reinterpret_cast<uint4*>(dst)[1] = b;
 }
 
+// Partial accumulators of split tiles: slot per CTA, [BN/16][128 rows][16]
+// fp32, so a warp's 16-column chunk is 2 KB contiguous.
+struct Partials {
+  const float* slots[4];  // contributors' slots, in CTA order
+  int n;
+  int row;                // row within the tile (0..127)
+};
+
+template <int BN>
+__device__ __forceinline__ const float* slot_chunk(const float* slot, int col, int row) {
+  return slot + (static_cast<int64_t>(col >> 4) * kBM + row) * 16;
+}
+
+// Load 16 accumulator columns starting at `col` and add the contributors'
+// partials (in order).
+template <int BN>
+__device__ __forceinline__ void load_acc16(uint32_t tacc, int col, const Partials& pp, float (&v)[16]) {
+  tmem_ld16(tacc + col, v);
+  for (int q = 0; q < pp.n; ++q) {
+    const float4* src = reinterpret_cast<const float4*>(slot_chunk<BN>(pp.slots[q], col, pp.row));
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float4 x = __ldcg(src + i);
+      v[4 * i] += x.x;
+      v[4 * i + 1] += x.y;
+      v[4 * i + 2] += x.z;
+      v[4 * i + 3] += x.w;
+    }
+  }
+}
+
 // Epilogue of one 128 x BN tile for the calling thread's row.
 template <int BN>
-__device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32_t tacc, int row, int M, int n0) {
+__device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32_t tacc, int row, int M, int n0,
+                                                  const Partials& pp) {
   const bool in_range = row < M;
   if (ep.mode == CORA_EPI_STORE_BF16) {
     uint16_t* crow = reinterpret_cast<uint16_t*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0;
 #pragma unroll 1
     for (int c = 0; c < BN; c += 16) {
       float v[16];
-      tmem_ld16(tacc + c, v);
+      load_acc16<BN>(tacc, c, pp, v);
       if (in_range) store_bf16x16(crow + c, v);
     }
   } else if (ep.mode == CORA_EPI_RESID_F32) {
@@ -67,7 +132,7 @@ __device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32
 #pragma unroll 1
     for (int c = 0; c < BN; c += 16) {
       float v[16];
-      tmem_ld16(tacc + c, v);
+      load_acc16<BN>(tacc, c, pp, v);
       if (in_range) {
         float4* p = reinterpret_cast<float4*>(crow + c);
 #pragma unroll
@@ -88,7 +153,8 @@ __device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32
 #pragma unroll 1
     for (int c = 0; c < BN / 2; c += 16) {
       float g[16], u[16];
-      tmem_ld16x2(tacc + c, tacc + BN / 2 + c, g, u);
+      load_acc16<BN>(tacc, c, pp, g);
+      load_acc16<BN>(tacc, BN / 2 + c, pp, u);
 #pragma unroll
       for (int j = 0; j < 16; ++j) g[j] = silu_f(g[j]) * u[j];
       if (in_range) store_bf16x16(crow + c, g);
@@ -104,7 +170,8 @@ __device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32
 #pragma unroll 1
       for (int j0 = 0; j0 < half; j0 += 16) {
         float x1[16], x2[16];
-        tmem_ld16x2(tacc + h0 + j0, tacc + h0 + half + j0, x1, x2);
+        load_acc16<BN>(tacc, h0 + j0, pp, x1);
+        load_acc16<BN>(tacc, h0 + half + j0, pp, x2);
         if (rot) {
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
@@ -123,10 +190,31 @@ __device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32
   }
 }
 
+__device__ __forceinline__ int ld_acquire(const int* p) {
+  int v;
+  asm volatile("ld.global.acquire.gpu.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Bounded spin until *flag != 0.
+__device__ __forceinline__ bool wait_flag(const int* flag, volatile int* abort, int* err) {
+  const long long t0 = clock64();
+  while (ld_acquire(flag) == 0) {
+    if (*abort) return false;
+    if (clock64() - t0 > CORA_WAIT_LIMIT) {
+      record_error(err, CORA_DERR_SPLIT_WAIT);
+      *abort = 1;
+      return false;
+    }
+    __nanosleep(100);
+  }
+  return true;
+}
+
 template <int BN>
 __global__ void __launch_bounds__(192, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
-                   int K, GemmEpilogue ep, int* err) {
+                   int K, GemmEpilogue ep, GemmWorkspace ws, int* err) {
   using Cfg = GemmCfg<BN>;
   constexpr int STAGES = Cfg::STAGES;
   constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN);
@@ -141,9 +229,11 @@ __global__ void __launch_bounds__(192, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int num_m = (M + kBM - 1) / kBM;
-  const int num_tiles = num_m * (N / BN);
-  const int kblocks = K / kBK;
+  const int num_n = N / BN;
+  const int num_tiles = ((M + kBM - 1) / kBM) * num_n;
+  const int KB = K / kBK;
+  const int W = num_tiles * KB;
+  const int G = gridDim.x;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -174,9 +264,11 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      for (int t = blockIdx.x; t < num_tiles; t += gridDim.x) {
-        const int mb = t % num_m, nb = t / num_m;
-        for (int kb = 0; kb < kblocks; ++kb) {
+      SegIter seg(blockIdx.x, G, W, KB);
+      int t, kb0, kb1;
+      while (seg.next(t, kb0, kb1)) {
+        const int mb = t / num_n, nb = t - mb * num_n;
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err, CORA_DERR_TMA_WAIT)) goto producer_done;
           uint8_t* sa = smem + stage * Cfg::STAGE_BYTES;
           mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
@@ -195,14 +287,17 @@ __global__ void __launch_bounds__(192, 1)
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
-      for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++it) {
+      SegIter seg(blockIdx.x, G, W, KB);
+      int t, kb0, kb1;
+      while (seg.next(t, kb0, kb1)) {
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
+        ++it;
         if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, err, CORA_DERR_MMA_WAIT)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         bool ok = true;
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(&full[stage], phase, abort_flag, err, CORA_DERR_MMA_WAIT)) {
             ok = false;
             break;
@@ -213,7 +308,7 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
             umma_bf16(d_tmem, sw128_kmajor_desc(a_addr + k * 32), sw128_kmajor_desc(b_addr + k * 32), IDESC,
-                      (kb | k) != 0);
+                      (kb > kb0 || k > 0) ? 1u : 0u);
           }
           umma_commit(&empty[stage]);
           if (++stage == STAGES) {
@@ -227,18 +322,67 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else {
     const int sub = warp & 3;  // TMEM sub-partition this warp may access
+    const int etid = threadIdx.x - 64;
+    const int row_local = sub * 32 + lane;
     int it = 0;
-    for (int t = blockIdx.x; t < num_tiles; t += gridDim.x, ++it) {
+    SegIter seg(blockIdx.x, G, W, KB);
+    int t, kb0, kb1;
+    while (seg.next(t, kb0, kb1)) {
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
-      if (!mbar_wait(&tfull[acc], acc_phase, abort_flag, err, CORA_DERR_EPI_WAIT)) break;
+      ++it;
+      const bool ok = mbar_wait(&tfull[acc], acc_phase, abort_flag, err, CORA_DERR_EPI_WAIT);
+      if (named_bar_or(1, 128, !ok)) break;  // uniform exit of the four epilogue warps
       tc_fence_after();
-      const int mb = t % num_m, nb = t / num_m;
-      const int row = mb * kBM + sub * 32 + lane;
+      const int mb = t / num_n, nb = t - mb * num_n;
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * BN;
-      gemm_epilogue_row<BN>(ep, tacc, row, M, nb * BN);
+      if (kb0 > 0) {
+        // Contributor: hand the partial accumulator to the tile's finisher.
+        float* slot = ws.partial + static_cast<int64_t>(blockIdx.x) * kBM * BN;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 16) {
+          float v[16];
+          tmem_ld16(tacc + c, v);
+          float4* dst = reinterpret_cast<float4*>(slot + (static_cast<int64_t>(c >> 4) * kBM + row_local) * 16);
+#pragma unroll
+          for (int i = 0; i < 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        }
+        tc_fence_before();
+        mbar_arrive(&tempty[acc]);
+        __threadfence();
+        named_bar_sync(1, 128);
+        if (etid == 0) atomicExch(ws.flags + blockIdx.x, 1);
+        continue;
+      }
+      Partials pp;
+      pp.n = 0;
+      pp.row = row_local;
+      int c_first = 0, c_last = -1;
+      if (kb1 < KB) {
+        // Finisher of a split tile: contributors are the next CTAs up to the
+        // one whose range holds the tile's last k-block.
+        const int last_it = t * KB + KB - 1;
+        c_first = blockIdx.x + 1;
+        c_last = c_first;
+        while (c_last + 1 < G && sk_start(c_last + 1, G, W) <= last_it) ++c_last;
+        bool fok = true;
+        if (etid == 0)
+          for (int c = c_first; c <= c_last && fok; ++c) fok = wait_flag(ws.flags + c, abort_flag, err);
+        if (named_bar_or(1, 128, !fok)) break;
+        for (int c = c_first; c <= c_last; ++c) {
+          (void)ld_acquire(ws.flags + c);
+          if (pp.n < 4) pp.slots[pp.n++] = ws.partial + static_cast<int64_t>(c) * kBM * BN;
+        }
+        if (c_last - c_first + 1 > 4) record_error(err, CORA_DERR_SPLIT_WAIT);  // cannot happen: grid checked
+      }
+      gemm_epilogue_row<BN>(ep, tacc, mb * kBM + row_local, M, nb * BN, pp);
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
+      if (c_last >= c_first) {
+        named_bar_sync(1, 128);  // every thread has read the partials
+        if (etid == 0)
+          for (int c = c_first; c <= c_last; ++c) atomicExch(ws.flags + c, 0);
+      }
     }
   }
 
@@ -259,13 +403,29 @@ int gemm_block_n(int N, int mode) {
   return (N % 256 == 0) ? 256 : 128;
 }
 
+size_t gemm_workspace_bytes(int num_sms) { return static_cast<size_t>(num_sms) * kBM * 256 * sizeof(float); }
+
+// Grid for a stream-K launch: one CTA per SM, but every CTA gets at least
+// ceil(KB/4) iterations, so a split tile has at most four contributors
+// besides its finisher; never more CTAs than iterations.
+static int gemm_grid(int M, int N, int K, int bn, int num_sms) {
+  const int tiles = ((M + kBM - 1) / kBM) * (N / bn);
+  const int KB = K / kBK;
+  const long long W = static_cast<long long>(tiles) * KB;
+  long long g = num_sms;
+  const long long max_by_share = W / ((KB + 3) / 4);
+  if (g > max_by_share) g = max_by_share;
+  if (g > W) g = W;
+  return g < 1 ? 1 : static_cast<int>(g);
+}
+
 template <int BN>
 static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K,
-                                  const GemmEpilogue& ep, int* err, int num_sms, cudaStream_t st) {
+                                  const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms,
+                                  cudaStream_t st) {
   using Cfg = GemmCfg<BN>;
-  const int tiles = ((M + kBM - 1) / kBM) * (N / BN);
-  const int grid = tiles < num_sms ? tiles : num_sms;
-  gemm_tc_kernel<BN><<<grid, 192, Cfg::SMEM_BYTES, st>>>(tmA, tmB, M, N, K, ep, err);
+  const int grid = gemm_grid(M, N, K, BN, num_sms);
+  gemm_tc_kernel<BN><<<grid, 192, Cfg::SMEM_BYTES, st>>>(tmA, tmB, M, N, K, ep, ws, err);
   return cudaGetLastError();
 }
 
@@ -278,7 +438,7 @@ cudaError_t gemm_prepare() {
 }
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, const GemmEpilogue& ep,
-                        int* err, int num_sms, cudaStream_t st) {
-  if (gemm_block_n(N, ep.mode) == 256) return launch_gemm_bn<256>(tmA, tmB, M, N, K, ep, err, num_sms, st);
-  return launch_gemm_bn<128>(tmA, tmB, M, N, K, ep, err, num_sms, st);
+                        const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st) {
+  if (gemm_block_n(N, ep.mode) == 256) return launch_gemm_bn<256>(tmA, tmB, M, N, K, ep, ws, err, num_sms, st);
+  return launch_gemm_bn<128>(tmA, tmB, M, N, K, ep, ws, err, num_sms, st);
 }

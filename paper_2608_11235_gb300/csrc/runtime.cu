@@ -56,6 +56,7 @@ struct DeviceCtx {
   int* err = nullptr;          // device error word for standalone ops
   void* scratch = nullptr;     // partials for standalone reductions
   size_t scratch_bytes = 0;
+  GemmWorkspace gemm_ws{nullptr, nullptr};  // stream-K workspace for cora_op_gemm
 };
 
 std::mutex g_mu;
@@ -72,6 +73,9 @@ int device_ctx(DeviceCtx** out) {
     CK(cudaDeviceGetAttribute(&c.num_sms, cudaDevAttrMultiProcessorCount, dev));
     CK(cudaMalloc(&c.err, sizeof(int)));
     CK(cudaMemset(c.err, 0, sizeof(int)));
+    CK(cudaMalloc(&c.gemm_ws.partial, gemm_workspace_bytes(c.num_sms)));
+    CK(cudaMalloc(&c.gemm_ws.flags, sizeof(int) * c.num_sms));
+    CK(cudaMemset(c.gemm_ws.flags, 0, sizeof(int) * c.num_sms));
     if (!g_encode) {
       cudaDriverEntryPointQueryResult q;
       void* fn = nullptr;
@@ -300,6 +304,7 @@ struct cora_session {
   int32_t* status = nullptr;   // device {all_done (byte 0), error word}
   int32_t* status_h = nullptr; // pinned host copy
   CUtensorMap tm_xn{}, tm_attn{}, tm_act{}, tm_xf{};
+  GemmWorkspace gemm_ws{nullptr, nullptr};
   cudaGraphExec_t graph = nullptr;
   int64_t batched_passes = 0;
   bool finished = false;
@@ -353,19 +358,19 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr) {
     REC(CORA_KIND_RMSNORM);
     GemmEpilogue e1{s->qkv, m->n_qkv, CORA_EPI_ROPE_BF16, s->rope, s->S, c.head_dim,
                     (c.n_heads + c.n_kv_heads) * c.head_dim};
-    CK(launch_gemm(s->tm_xn, m->tm_qkv[l], M, m->n_qkv, d, e1, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_xn, m->tm_qkv[l], M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_QKV);
     launch_attention(s->qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, st);
     REC(CORA_KIND_ATTENTION);
     GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0};
-    CK(launch_gemm(s->tm_attn, m->tm_o[l], M, d, c.n_heads * c.head_dim, e2, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_attn, m->tm_o[l], M, d, c.n_heads * c.head_dim, e2, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_O);
     launch_rmsnorm(s->h, m->ffn_norm[l], s->xn, M, d, c.norm_eps, st);
     REC(CORA_KIND_RMSNORM);
     GemmEpilogue e3{s->act, m->f_pad, CORA_EPI_SWIGLU, nullptr, 0, 0, 0};
-    CK(launch_gemm(s->tm_xn, m->tm_gu[l], M, 2 * m->f_pad, d, e3, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_xn, m->tm_gu[l], M, 2 * m->f_pad, d, e3, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_GATE_UP);
-    CK(launch_gemm(s->tm_act, m->tm_down[l], M, d, m->f_pad, e2, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_act, m->tm_down[l], M, d, m->f_pad, e2, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_DOWN);
   }
   launch_final_norm_rows(s->h, m->final_norm, s->ctrl, s->xf, s->B, s->S, s->P, s->BL, s->n_blocks, d, c.norm_eps,
@@ -451,6 +456,9 @@ extern "C" int cora_session_create(cora_model* m, int32_t batch, const int32_t* 
   SK(sess_alloc(s, size_t(s->R), &s->unmask));
   SK(sess_alloc(s, size_t(s->R), &s->accept));
   SK(sess_alloc(s, 4, &s->status));
+  SK(sess_alloc(s, gemm_workspace_bytes(m->num_sms) / sizeof(float), &s->gemm_ws.partial));
+  SK(sess_alloc(s, size_t(m->num_sms), &s->gemm_ws.flags));
+  if (cudaMemset(s->gemm_ws.flags, 0, sizeof(int) * m->num_sms) != cudaSuccess) SK(fail(CORA_ECUDA, "memset"));
   {
     void* hp = nullptr;
     if (cudaHostAlloc(&hp, 16, cudaHostAllocDefault) != cudaSuccess) SK(fail(CORA_ENOMEM, "pinned alloc"));
@@ -716,7 +724,7 @@ extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32
   if (!make_tmap_bf16_2d(&ta, A, M, K, size_t(K) * 2, 128, 64) || !make_tmap_bf16_2d(&tb, B, N, K, size_t(K) * 2, bn, 64))
     return fail(CORA_ECUDA, "cora_op_gemm: tensor map encoding failed");
   GemmEpilogue ep{C, ldc, epilogue, rope, seq, head_dim, rope_cols};
-  CK(launch_gemm(ta, tb, M, N, K, ep, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
+  CK(launch_gemm(ta, tb, M, N, K, ep, dc->gemm_ws, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
   return CORA_OK;
 }
 

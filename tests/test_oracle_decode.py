@@ -42,10 +42,22 @@ def test_accept_all_one_pass_per_block(model, prompt):
         assert np.array_equal(s["after"].tokens, s["x_hat"])
 
 
-def test_persistence_one_two_passes_per_block(model, prompt):
+def test_accept_all_with_one_persistence_check(model, prompt):
+    """delta_p = 0, m = 1: nothing is accepted on a block's first pass; after
+    that a block ends at the first pass on which every position still
+    unresolved (and not transferred) repeats its previous prediction."""
     cfg, w = model
-    tr = O.generate(cfg, w, prompt, G, BL, T, 0.0, 1)
-    assert tr.passes_per_block == [2] * (G // BL)
+    tr = O.generate(cfg, w, prompt, G, BL, T, 0.0, 1, record=True)
+    assert all(2 <= p <= T for p in tr.passes_per_block)
+    for s in tr.steps:
+        r = s["result"]
+        U = s["before"].state == O.UNRESOLVED
+        if s["step"] == 0:
+            assert not r.accepted
+            continue
+        rest = [i for i in np.flatnonzero(U) if i not in r.transferred]
+        stable = all(s["before"].prev[i] == s["x_hat"][i] for i in rest)
+        assert r.done == stable
 
 
 @pytest.mark.parametrize("tau,K", [(0.3, 1), (0.5, 0), (0.2, 2), (0.65, 1)])
