@@ -52,20 +52,52 @@ __device__ __forceinline__ int sk_start(int c, int G, int W) {
   return static_cast<int>((static_cast<long long>(c) * W) / G);
 }
 
-// Walks a CTA's iteration range as segments (tile, kb0, kb1).
+// A CTA's iteration range as segments (tile, kb0, kb1), visited in the order
+// (1) its first segment (a contributor when it starts mid-tile), (2) its
+// last segment (a split tile it finishes when it ends mid-tile), (3) the
+// whole tiles in between.  Putting both split segments first lets their
+// hand-off and fix-up overlap the MMAs of the whole tiles.
 struct SegIter {
-  int it, it_end, kb_per_tile;
-  __device__ SegIter(int c, int G, int W, int KB) : it(sk_start(c, G, W)), it_end(sk_start(c + 1, G, W)),
-                                                     kb_per_tile(KB) {}
+  int it0, it1, kb_per_tile, t_first, t_last, idx;
+  __device__ SegIter(int c, int G, int W, int KB)
+      : it0(sk_start(c, G, W)), it1(sk_start(c + 1, G, W)), kb_per_tile(KB), idx(0) {
+    t_first = it0 / KB;
+    t_last = it1 > it0 ? (it1 - 1) / KB : t_first - 1;
+  }
   __device__ bool next(int& t, int& kb0, int& kb1) {
-    if (it >= it_end) return false;
-    t = it / kb_per_tile;
-    kb0 = it - t * kb_per_tile;
-    kb1 = min(kb_per_tile, kb0 + (it_end - it));
-    it += kb1 - kb0;
+    if (it1 <= it0) return false;
+    const int KB = kb_per_tile;
+    if (t_first == t_last) {  // the whole range lies in one tile
+      if (idx++ > 0) return false;
+      t = t_first;
+      kb0 = it0 - t * KB;
+      kb1 = it1 - t * KB;
+      return true;
+    }
+    const int n_mid = t_last - t_first - 1;
+    if (idx >= 2 + n_mid) return false;
+    if (idx == 0) {
+      t = t_first;
+      kb0 = it0 - t * KB;
+      kb1 = KB;
+    } else if (idx == 1) {
+      t = t_last;
+      kb0 = 0;
+      kb1 = it1 - t * KB;
+    } else {
+      t = t_first + idx - 1;
+      kb0 = 0;
+      kb1 = KB;
+    }
+    ++idx;
     return true;
   }
 };
+
+__device__ __forceinline__ void red_add_v4(float* dst, const float* a) {
+  asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst), "f"(a[0]), "f"(a[1]), "f"(a[2]), "f"(a[3])
+               : "memory");
+}
 
 __device__ __forceinline__ float silu_f(float x) { return x / (1.f + __expf(-x)); }
 
@@ -91,30 +123,62 @@ struct Partials {
   int row;                // row within the tile (0..127)
 };
 
-template <int BN>
-__device__ __forceinline__ const float* slot_chunk(const float* slot, int col, int row) {
-  return slot + (static_cast<int64_t>(col >> 4) * kBM + row) * 16;
+__device__ __forceinline__ const float4* slot_chunk(const float* slot, int col, int row) {
+  return reinterpret_cast<const float4*>(slot + (static_cast<int64_t>(col >> 4) * kBM + row) * 16);
 }
 
-// Load 16 accumulator columns starting at `col` and add the contributors'
-// partials (in order).
-template <int BN>
-__device__ __forceinline__ void load_acc16(uint32_t tacc, int col, const Partials& pp, float (&v)[16]) {
-  tmem_ld16(tacc + col, v);
-  for (int q = 0; q < pp.n; ++q) {
-    const float4* src = reinterpret_cast<const float4*>(slot_chunk<BN>(pp.slots[q], col, pp.row));
+// Loads four 16-column accumulator chunks (columns col[0..3]) under one TMEM
+// wait, then adds every contributor's partial; all global loads of one
+// contributor are issued before any is used, so the epilogue pays one memory
+// round trip per four chunks instead of one per chunk.
+__device__ __forceinline__ void load_acc64(uint32_t tacc, const int (&col)[4], const Partials& pp,
+                                           float (&v)[4][16]) {
+  uint32_t r[64];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%64];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, "
+      "[%65];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47}, "
+      "[%66];\n\t"
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, "
+      "[%67];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+        "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]),
+        "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]),
+        "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(tacc + col[0]), "r"(tacc + col[1]), "r"(tacc + col[2]), "r"(tacc + col[3])
+      : "memory");
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const float4 x = __ldcg(src + i);
-      v[4 * i] += x.x;
-      v[4 * i + 1] += x.y;
-      v[4 * i + 2] += x.z;
-      v[4 * i + 3] += x.w;
+  for (int q = 0; q < 4; ++q)
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[q][i] = __uint_as_float(r[16 * q + i]);
+  for (int p = 0; p < pp.n; ++p) {
+    float4 x[4][4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float4* src = slot_chunk(pp.slots[p], col[q], pp.row);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) x[q][i] = __ldcg(src + i);
     }
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        v[q][4 * i] += x[q][i].x;
+        v[q][4 * i + 1] += x[q][i].y;
+        v[q][4 * i + 2] += x[q][i].z;
+        v[q][4 * i + 3] += x[q][i].w;
+      }
   }
 }
 
-// Epilogue of one 128 x BN tile for the calling thread's row.
+// Epilogue of one 128 x BN tile for the calling thread's row, 64 columns
+// (four chunks) per step.
 template <int BN>
 __device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32_t tacc, int row, int M, int n0,
                                                   const Partials& pp) {
@@ -122,44 +186,46 @@ __device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32
   if (ep.mode == CORA_EPI_STORE_BF16) {
     uint16_t* crow = reinterpret_cast<uint16_t*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0;
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 16) {
-      float v[16];
-      load_acc16<BN>(tacc, c, pp, v);
-      if (in_range) store_bf16x16(crow + c, v);
+    for (int c = 0; c < BN; c += 64) {
+      float v[4][16];
+      const int cols[4] = {c, c + 16, c + 32, c + 48};
+      load_acc64(tacc, cols, pp, v);
+      if (in_range)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) store_bf16x16(crow + c + 16 * q, v[q]);
     }
   } else if (ep.mode == CORA_EPI_RESID_F32) {
+    // h += acc as vector reductions performed at L2: no read round trip, and
+    // exactly one add per element per launch, so the result is deterministic.
     float* crow = reinterpret_cast<float*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0;
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 16) {
-      float v[16];
-      load_acc16<BN>(tacc, c, pp, v);
-      if (in_range) {
-        float4* p = reinterpret_cast<float4*>(crow + c);
+    for (int c = 0; c < BN; c += 64) {
+      float v[4][16];
+      const int cols[4] = {c, c + 16, c + 32, c + 48};
+      load_acc64(tacc, cols, pp, v);
+      if (in_range)
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          float4 h = p[q];
-          h.x += v[4 * q];
-          h.y += v[4 * q + 1];
-          h.z += v[4 * q + 2];
-          h.w += v[4 * q + 3];
-          p[q] = h;
-        }
-      }
+        for (int i = 0; i < 16; ++i) red_add_v4(crow + c + 4 * i, &v[i >> 2][(i & 3) * 4]);
     }
   } else if (ep.mode == CORA_EPI_SWIGLU) {
     // Tile columns [0, BN/2) are gate rows, [BN/2, BN) the matching up rows
     // of output features n0/2 .. n0/2 + BN/2.
     uint16_t* crow = reinterpret_cast<uint16_t*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0 / 2;
 #pragma unroll 1
-    for (int c = 0; c < BN / 2; c += 16) {
-      float g[16], u[16];
-      load_acc16<BN>(tacc, c, pp, g);
-      load_acc16<BN>(tacc, BN / 2 + c, pp, u);
+    for (int c = 0; c < BN / 2; c += 32) {
+      float v[4][16];
+      const int cols[4] = {c, c + 16, BN / 2 + c, BN / 2 + c + 16};
+      load_acc64(tacc, cols, pp, v);
 #pragma unroll
-      for (int j = 0; j < 16; ++j) g[j] = silu_f(g[j]) * u[j];
-      if (in_range) store_bf16x16(crow + c, g);
+      for (int q = 0; q < 2; ++q)
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[q][j] = silu_f(v[q][j]) * v[q + 2][j];
+      if (in_range) {
+        store_bf16x16(crow + c, v[0]);
+        store_bf16x16(crow + c + 16, v[1]);
+      }
     }
-  } else {  // CORA_EPI_ROPE_BF16
+  } else {  // CORA_EPI_ROPE_BF16: rotate pairs (j, j + hd/2) of every head
     uint16_t* crow = reinterpret_cast<uint16_t*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0;
     const int hd = ep.head_dim, half = hd / 2;
     const int pos = in_range ? row % ep.seq : 0;
@@ -168,22 +234,26 @@ __device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32
     for (int h0 = 0; h0 < BN; h0 += hd) {
       const bool rot = n0 + h0 < ep.rope_cols;
 #pragma unroll 1
-      for (int j0 = 0; j0 < half; j0 += 16) {
-        float x1[16], x2[16];
-        load_acc16<BN>(tacc, h0 + j0, pp, x1);
-        load_acc16<BN>(tacc, h0 + half + j0, pp, x2);
+      for (int j0 = 0; j0 < half; j0 += 32) {
+        float v[4][16];
+        const int cols[4] = {h0 + j0, h0 + j0 + 16, h0 + half + j0, h0 + half + j0 + 16};
+        load_acc64(tacc, cols, pp, v);
         if (rot) {
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const float2 cs = tab[j0 + j];
-            const float a = x1[j], b = x2[j];
-            x1[j] = a * cs.x - b * cs.y;
-            x2[j] = b * cs.x + a * cs.y;
-          }
+          for (int q = 0; q < 2; ++q)
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
+              const float2 cs = tab[j0 + 16 * q + j];
+              const float a = v[q][j], b = v[q + 2][j];
+              v[q][j] = a * cs.x - b * cs.y;
+              v[q + 2][j] = b * cs.x + a * cs.y;
+            }
         }
         if (in_range) {
-          store_bf16x16(crow + h0 + j0, x1);
-          store_bf16x16(crow + h0 + half + j0, x2);
+          store_bf16x16(crow + h0 + j0, v[0]);
+          store_bf16x16(crow + h0 + j0 + 16, v[1]);
+          store_bf16x16(crow + h0 + half + j0, v[2]);
+          store_bf16x16(crow + h0 + half + j0 + 16, v[3]);
         }
       }
     }
@@ -339,13 +409,21 @@ __global__ void __launch_bounds__(192, 1)
       if (kb0 > 0) {
         // Contributor: hand the partial accumulator to the tile's finisher.
         float* slot = ws.partial + static_cast<int64_t>(blockIdx.x) * kBM * BN;
+        Partials none;
+        none.n = 0;
+        none.row = row_local;
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 16) {
-          float v[16];
-          tmem_ld16(tacc + c, v);
-          float4* dst = reinterpret_cast<float4*>(slot + (static_cast<int64_t>(c >> 4) * kBM + row_local) * 16);
+        for (int c = 0; c < BN; c += 64) {
+          float v[4][16];
+          const int cols[4] = {c, c + 16, c + 32, c + 48};
+          load_acc64(tacc, cols, none, v);
 #pragma unroll
-          for (int i = 0; i < 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+          for (int q = 0; q < 4; ++q) {
+            float4* dst = reinterpret_cast<float4*>(slot + (static_cast<int64_t>((c >> 4) + q) * kBM + row_local) * 16);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              dst[i] = make_float4(v[q][4 * i], v[q][4 * i + 1], v[q][4 * i + 2], v[q][4 * i + 3]);
+          }
         }
         tc_fence_before();
         mbar_arrive(&tempty[acc]);
