@@ -201,6 +201,49 @@ def kernel_costs(cfg: dict):
     }
 
 
+def gate_isolation(peaks, reps: int = 5):
+    """Eq. 1 from materialised bf16 logits [B, 32, 126464] + transfer rule +
+    gate (cora_reduce_gate), B in {1, 8, 64}; HBM-bound.  L2 is flushed
+    (a 256 MB write) before every timed launch; CUDA events bracket the launch
+    only."""
+    import torch
+
+    from paper_2608_11235_gb300 import configs, cora, synth
+
+    gi = configs.GATE_ISOLATION
+    R, V = gi["rows"], gi["vocab"]
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    out = {}
+    for B in gi["batches"]:
+        hist = synth.gate_history(gi["seed"], B, R, V, gi["n_hist"], gi["keep"])
+        lg = torch.from_numpy(synth.gate_logits_bf16(gi["seed"], B, R, V, hist[-1], gi["keep"]).view(np.int16)).cuda()
+        st = lambda dt: torch.zeros((B, R), dtype=dt, device="cuda")
+        conf, arg, prev, persist = st(torch.float32), st(torch.int32), st(torch.int32), st(torch.int32)
+        state, tokens, unmask, accept = st(torch.uint8), st(torch.int32), st(torch.uint8), st(torch.uint8)
+        done = torch.zeros(B, dtype=torch.uint8, device="cuda")
+        ts = []
+        for i in range(reps + 2):
+            flush.fill_(i & 0xFF)
+            prev.fill_(-1)
+            persist.zero_()
+            state.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            cora.cora_reduce_gate(lg, B, R, V, conf, arg, prev, persist, state, tokens, gi["k_step"], gi["tau"],
+                                  gi["K"], unmask, accept, done)
+            e1.record()
+            e1.synchronize()
+            if i >= 2:
+                ts.append(e0.elapsed_time(e1))
+        ms = statistics.median(ts)
+        nbytes = B * R * V * 2
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        out[f"B{B}"] = {"us": round(ms * 1e3, 2), "GB_s": round(gbs, 1),
+                        "frac": round(gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]), 4), "bytes": nbytes}
+        del lg
+    return out
+
+
 def run_cora(args, cfg, ws, rank, local):
     import torch
 
@@ -318,6 +361,7 @@ def run_cora(args, cfg, ws, rank, local):
     if s is not None:
         cora.cora_session_destroy(s)
     cora.cora_model_destroy(m)
+    gate_iso = None if args.no_variant else gate_isolation(peaks)
 
     value = ws * B * G * args.steps / (ms * 1e-3)
     launches_per_pass = 4 + 7 * cfg["n_layers"]
@@ -343,6 +387,7 @@ def run_cora(args, cfg, ws, rank, local):
         "gpu_launches": int(total_passes * launches_per_pass + args.steps),
         "clocks": clocks,
         "gate_exercising": gx,
+        "gate_isolation": gate_iso,
     }
     return result, float(per_seq_passes.mean())
 
