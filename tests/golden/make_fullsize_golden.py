@@ -1,0 +1,70 @@
+"""Writes the oracle's first-step results for the 8B-class workloads.
+
+For each workload, sequence 0's first executed step (block 0, step 0: canvas
+= prompt + all masks) is computed by the CPU oracle in float64, one layer at
+a time (weights regenerated per layer by the seeded generator), then Eq. 1 on
+the 32 active rows for two LM heads: the workload's own head and the
+gate-exercising head N(0, 8/sqrt(d)).  Only oracle/ and the seeded input
+generator are called.
+
+    python tests/golden/make_fullsize_golden.py [preset ...]
+
+Output: tests/golden/fullsize_<preset>.json (conf, argmax, top-1/top-2
+probability margin and logit gap per row, for each head).
+"""
+
+from __future__ import annotations
+
+import json
+import os
+import sys
+import time
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, os.path.dirname(os.path.dirname(HERE)))
+
+from oracle import cora_oracle as O  # noqa: E402
+from paper_2608_11235_gb300 import configs, synth  # noqa: E402
+
+PRESETS = ["llada8b-shape-256+256", "dream7b-shape-256+512-b4", "llada8b-shape-512+1024-b8"]
+
+
+def head_eq1(cfg, rows, v_chunk=16384):
+    V = cfg["vocab"]
+    logits = np.empty((rows.shape[0], V))
+    for v0 in range(0, V, v_chunk):
+        v1 = min(V, v0 + v_chunk)
+        head = {"final_norm": np.ones(cfg["d_model"]),
+                "lm_head": synth.weight_f64(cfg, -1, synth.LM_HEAD, slice(v0, v1))}
+        logits[:, v0:v1] = O.lm_logits(cfg, head, rows)
+    c, a = O.top1(logits)
+    srt = np.sort(logits, axis=-1)
+    return {"conf": c.tolist(), "argmax": a.tolist(), "margin": O.top2_margin(logits).tolist(),
+            "logit_gap": (srt[:, -1] - srt[:, -2]).tolist()}
+
+
+def run(preset: str) -> None:
+    cfg = dict(configs.PRESETS[preset])
+    P, G, BL = cfg["prompt_len"], cfg["gen_len"], cfg["block_len"]
+    prompt = synth.prompts(cfg["prompt_seed"], cfg["batch"], P, cfg["mask_id"])[0]
+    x = np.concatenate([prompt, np.full(G, cfg["mask_id"])])
+    h = np.stack([synth.weight_f64(cfg, -1, synth.EMBED, slice(int(t), int(t) + 1))[0] for t in x])
+    pos = np.arange(len(x))
+    t0 = time.time()
+    for l in range(cfg["n_layers"]):
+        h = O.layer_forward(cfg, synth.layer_weights_f64(cfg, l), h, pos)
+        print(f"{preset}: layer {l} done at {time.time() - t0:.0f} s", flush=True)
+    rows = h[P: P + BL]
+    out = {"preset": preset, "sequence": 0, "block": 0, "step": 0,
+           "source": "oracle/cora_oracle.py (layer_forward, lm_logits, top1, top2_margin), float64",
+           "heads": {"workload": head_eq1(cfg, rows),
+                     "gate_exercising": head_eq1(configs.gate_exercising(cfg), rows)}}
+    with open(os.path.join(HERE, f"fullsize_{preset}.json"), "w") as f:
+        json.dump(out, f)
+
+
+if __name__ == "__main__":
+    for p in (sys.argv[1:] or PRESETS):
+        run(p)
