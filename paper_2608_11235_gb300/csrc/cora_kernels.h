@@ -45,16 +45,29 @@ void launch_rmsnorm(const float* x, const uint16_t* w, uint16_t* out, int M, int
 void launch_final_norm_rows(const float* h, const uint16_t* w, const int32_t* ctrl, uint16_t* out, int B, int S,
                             int P, int BL, int n_blocks, int d, float eps, cudaStream_t st);
 
-// Eq. 1 partials from materialised bf16 logits [rows, V]: grid (n_chunks, rows).
+// Gate buffers of B blocks of R positions ([B, R] each; done is [B]).
+struct GateBuffers {
+  float* conf;
+  int32_t* argmax;
+  int32_t* prev;
+  int32_t* persist;
+  uint8_t* state;
+  int32_t* tokens;
+  uint8_t* unmask;
+  uint8_t* accept;
+  uint8_t* done;
+};
+
+// Eq. 1 from materialised bf16 logits [rows, V], grid (n_chunks, rows), with
+// the combine (and, when gate is set, the transfer rule + Eq. 2-4 of each
+// block of R rows) done by the last CTA of each group.  counters: zeroed ints,
+// one per row (gate == false) or per block (gate == true); left zeroed.
 int reduce_top1_parts_count(int rows, int V, int num_sms);
-void launch_reduce_top1_parts(const uint16_t* logits, int rows, int V, int n_chunks, Top1Part* parts,
-                              cudaStream_t st);
+void launch_reduce_fused(const uint16_t* logits, int rows, int V, int n_chunks, Top1Part* parts, int* counters,
+                         const GateBuffers& gb, int R, int k, float tau, int K, bool gate, cudaStream_t st);
 void launch_combine_top1(const Top1Part* parts, int n_parts, int rows, float* conf, int32_t* argmax,
                          cudaStream_t st);
-void launch_gate_transfer(const Top1Part* parts, int n_parts, const float* conf_in, const int32_t* argmax_in,
-                          float* conf_out, int32_t* argmax_out, int32_t* prev, int32_t* persist, uint8_t* state,
-                          int32_t* tokens, int B, int R, int k, float tau, int K, uint8_t* unmask, uint8_t* accept,
-                          uint8_t* done, cudaStream_t st);
+void launch_gate_transfer(const GateBuffers& gb, int B, int R, int k, float tau, int K, cudaStream_t st);
 void launch_session_gate(const SessionGateArgs& a, cudaStream_t st);
 
 // GEMM (tcgen05).  Epilogue parameters.

@@ -26,70 +26,77 @@ __device__ __forceinline__ Top1 warp_merge(Top1 st) {
 }
 
 // ---------------------------------------------------------------- Eq. 1 (K9)
-// Block (c, row) reduces logits[row, c*chunk : (c+1)*chunk] into one partial.
-__global__ void __launch_bounds__(256) reduce_top1_parts_kernel(const uint16_t* __restrict__ logits, int rows, int V,
-                                                                int chunk, Top1Part* __restrict__ parts) {
-  const int row = blockIdx.y, c = blockIdx.x;
-  const int lo = c * chunk;
-  const int hi = min(V, lo + chunk);
-  const uint16_t* p = logits + static_cast<int64_t>(row) * V;
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Adds 8 bf16 logits (one 16-byte word, ids i0 .. i0+7) to a running Top1
+// state.  The running max changes rarely, so the common path is a max tree,
+// then exp2 terms against the unchanged max.
+__device__ __forceinline__ void top1_add8(Top1& st, uint4 u, int i0) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  float v[8];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    v[2 * j] = __uint_as_float(w[j] << 16);
+    v[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
+  }
+  const float mv = fmaxf(fmaxf(fmaxf(v[0], v[1]), fmaxf(v[2], v[3])), fmaxf(fmaxf(v[4], v[5]), fmaxf(v[6], v[7])));
+  if (mv > st.m) {  // new running max: first id attaining it, rescale the sum
+    int mi = 7;
+#pragma unroll
+    for (int j = 6; j >= 0; --j)
+      if (v[j] == mv) mi = j;
+    st.s *= ex2_approx((st.m - mv) * kLog2e);
+    st.m = mv;
+    st.idx = i0 + mi;
+  }
+  const float mL = st.m * kLog2e;
+  float acc = 0.f;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) acc += ex2_approx(fmaf(v[j], kLog2e, -mL));
+  st.s += acc;
+}
+
+// Partial of logits[row, lo:hi]; block-wide result valid in thread 0.
+__device__ __forceinline__ Top1 reduce_range(const uint16_t* __restrict__ p, int lo, int hi, bool vec) {
   Top1 st = top1_empty();
-  if ((V & 7) == 0) {
-    for (int i = lo + threadIdx.x * 8; i < hi; i += blockDim.x * 8) {
-      const uint4 u = __ldcs(reinterpret_cast<const uint4*>(p + i));
-      const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-      float v[8];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        v[2 * j] = __uint_as_float(w[j] << 16);
-        v[2 * j + 1] = __uint_as_float(w[j] & 0xFFFF0000u);
-      }
-      float mv = v[0];
-      int mi = 0;
-#pragma unroll
-      for (int j = 1; j < 8; ++j)
-        if (v[j] > mv) {
-          mv = v[j];
-          mi = j;
-        }
-      if (mv > st.m) {
-        st.s *= exp2f((st.m - mv) * kLog2e);
-        st.m = mv;
-        st.idx = i + mi;
-      }
-      float acc = 0.f;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) acc += exp2f((v[j] - st.m) * kLog2e);
-      st.s += acc;
+  if (vec) {
+    const uint4* pv = reinterpret_cast<const uint4*>(p);
+    const int stride = blockDim.x * 8;
+    int i = lo + threadIdx.x * 8;
+    for (; i + 3 * stride < hi; i += 4 * stride) {  // four 16-byte loads in flight per thread
+      const uint4 a = __ldcs(pv + (i >> 3));
+      const uint4 b = __ldcs(pv + ((i + stride) >> 3));
+      const uint4 c = __ldcs(pv + ((i + 2 * stride) >> 3));
+      const uint4 d = __ldcs(pv + ((i + 3 * stride) >> 3));
+      top1_add8(st, a, i);
+      top1_add8(st, b, i + stride);
+      top1_add8(st, c, i + 2 * stride);
+      top1_add8(st, d, i + 3 * stride);
     }
+    for (; i < hi; i += stride) top1_add8(st, __ldcs(pv + (i >> 3)), i);
   } else {
     for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) {
       const float v = bf16_bits_to_float(p[i]);
       if (v > st.m) {
-        st.s *= exp2f((st.m - v) * kLog2e);
+        st.s *= ex2_approx((st.m - v) * kLog2e);
         st.m = v;
         st.idx = i;
       }
-      st.s += exp2f((v - st.m) * kLog2e);
+      st.s += ex2_approx((v - st.m) * kLog2e);
     }
   }
   st = warp_merge(st);
-  __shared__ Top1 wpart[8];
+  __shared__ Top1 wpart[32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (lane == 0) wpart[warp] = st;
   __syncthreads();
   if (warp == 0) {
     st = lane < static_cast<int>(blockDim.x >> 5) ? wpart[lane] : top1_empty();
     st = warp_merge(st);
-    if (lane == 0) parts[static_cast<int64_t>(c) * rows + row] = Top1Part{st.m, st.s, st.idx};
-  }
-}
-
-__device__ __forceinline__ Top1 combine_parts(const Top1Part* __restrict__ parts, int n_parts, int rows, int row) {
-  Top1 st = top1_empty();
-  for (int q = 0; q < n_parts; ++q) {
-    const Top1Part pp = parts[static_cast<int64_t>(q) * rows + row];
-    st = top1_merge(st, Top1{pp.m, pp.s, pp.idx});
   }
   return st;
 }
@@ -101,7 +108,8 @@ __device__ __forceinline__ Top1 warp_combine_parts(const Top1Part* __restrict__ 
   const int lane = threadIdx.x & 31;
   Top1 st = top1_empty();
   for (int q = lane; q < n_parts; q += 32) {
-    const Top1Part pp = parts[static_cast<int64_t>(q) * rows + row];
+    const Top1Part* src = parts + static_cast<int64_t>(q) * rows + row;
+    const Top1Part pp{__ldcg(&src->m), __ldcg(&src->s), __ldcg(&src->idx)};
     st = top1_merge(st, Top1{pp.m, pp.s, pp.idx});
   }
   return warp_merge(st);
@@ -162,45 +170,89 @@ __device__ __forceinline__ bool gate_warp(GateLane& g, bool valid, int k, float 
   return __ballot_sync(0xffffffffu, valid && g.state == CORA_UNRESOLVED) == 0u;
 }
 
-// Standalone gate on [B, R] buffers; conf/argmax come from `parts` when given,
-// else from conf_in / argmax_in.
-__global__ void gate_transfer_kernel(const Top1Part* __restrict__ parts, int n_parts,
-                                     const float* __restrict__ conf_in, const int32_t* __restrict__ argmax_in,
-                                     float* __restrict__ conf_out, int32_t* __restrict__ argmax_out, int32_t* prev,
-                                     int32_t* persist, uint8_t* state, int32_t* tokens, int B, int R, int k,
-                                     float tau, int K, uint8_t* unmask, uint8_t* accept, uint8_t* done) {
-  const int b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (b >= B) return;  // warp-uniform
+// Gate of block b on [B, R] buffers by one warp (conf/argmax already known).
+__device__ __forceinline__ void gate_block(const GateBuffers& gb, int b, int R, int k, float tau, int K) {
   const int lane = threadIdx.x & 31;
   const bool valid = lane < R;
   const int64_t e = static_cast<int64_t>(b) * R + lane;
   GateLane g{};
   if (valid) {
-    if (parts) {
-      const Top1 st = combine_parts(parts, n_parts, B * R, static_cast<int>(e));
-      g.c = 1.f / st.s;
-      g.xhat = st.idx;
-      if (conf_out) conf_out[e] = g.c;
-      if (argmax_out) argmax_out[e] = g.xhat;
-    } else {
-      g.c = conf_in[e];
-      g.xhat = argmax_in[e];
-    }
-    g.prev = prev[e];
-    g.persist = persist[e];
-    g.state = state[e];
-    g.token = tokens[e];
+    g.c = gb.conf[e];
+    g.xhat = gb.argmax[e];
+    g.prev = gb.prev[e];
+    g.persist = gb.persist[e];
+    g.state = gb.state[e];
+    g.token = gb.tokens[e];
   }
   const bool blk_done = gate_warp(g, valid, k, tau, K);
   if (valid) {
-    prev[e] = g.prev;
-    persist[e] = g.persist;
-    state[e] = static_cast<uint8_t>(g.state);
-    tokens[e] = g.token;
-    unmask[e] = g.T;
-    accept[e] = g.A;
+    gb.prev[e] = g.prev;
+    gb.persist[e] = g.persist;
+    gb.state[e] = static_cast<uint8_t>(g.state);
+    gb.tokens[e] = g.token;
+    gb.unmask[e] = g.T;
+    gb.accept[e] = g.A;
   }
-  if (lane == 0) done[b] = blk_done;
+  if (lane == 0) gb.done[b] = blk_done;
+}
+
+// Standalone gate on [B, R] buffers (conf/argmax given), one warp per block.
+__global__ void gate_transfer_kernel(GateBuffers gb, int B, int R, int k, float tau, int K) {
+  const int b = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (b >= B) return;  // warp-uniform
+  gate_block(gb, b, R, k, tau, K);
+}
+
+// Eq. 1 over logits [rows, V] in chunks, fused with what follows.  Block
+// (c, row) reduces one chunk to a partial; the last block to finish a group
+// (a row, or with the gate a whole block of R rows) combines the group's
+// partials in chunk order and then either writes conf/argmax (gate == false)
+// or also runs the transfer rule and Eq. 2-4 for that block.  Completion is
+// counted with one atomic per block (no waiting); the last block resets the
+// counter, so consecutive launches reuse it.
+__global__ void __launch_bounds__(256) reduce_fused_kernel(const uint16_t* __restrict__ logits, int rows, int V,
+                                                           int chunk, int n_chunks, Top1Part* __restrict__ parts,
+                                                           int* __restrict__ counters, GateBuffers gb, int R, int k,
+                                                           float tau, int K, int gate) {
+  const int row = blockIdx.y, c = blockIdx.x;
+  const int lo = c * chunk;
+  const int hi = min(V, lo + chunk);
+  const Top1 st = reduce_range(logits + static_cast<int64_t>(row) * V, lo, hi, (V & 7) == 0);
+  __shared__ int is_last;
+  if (threadIdx.x == 0) {
+    parts[static_cast<int64_t>(c) * rows + row] = Top1Part{st.m, st.s, st.idx};
+    __threadfence();
+    const int grp = gate ? row / R : row;
+    const int total = gate ? R * n_chunks : n_chunks;
+    const int old = atomicAdd(counters + grp, 1);
+    is_last = old == total - 1;
+    if (is_last) counters[grp] = 0;
+  }
+  __syncthreads();
+  if (!is_last) return;  // uniform per block
+  __threadfence();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  if (!gate) {
+    if (warp == 0) {
+      const Top1 t = warp_combine_parts(parts, n_chunks, rows, row);
+      if (lane == 0) {
+        gb.conf[row] = 1.f / t.s;  // max_v softmax = exp(m - m) / sum exp(l - m)
+        gb.argmax[row] = t.idx;
+      }
+    }
+    return;
+  }
+  const int b = row / R;
+  for (int r = warp; r < R; r += nw) {
+    const Top1 t = warp_combine_parts(parts, n_chunks, rows, b * R + r);
+    if (lane == 0) {
+      gb.conf[b * R + r] = 1.f / t.s;
+      gb.argmax[b * R + r] = t.idx;
+    }
+  }
+  __threadfence_block();
+  __syncthreads();
+  if (warp == 0) gate_block(gb, b, R, k, tau, K);
 }
 
 // Session gate: one CTA, warps stride over sequences.  Each unfinished
@@ -286,27 +338,24 @@ int reduce_top1_parts_count(int rows, int V, int num_sms) {
   return n < 1 ? 1 : n;
 }
 
-void launch_reduce_top1_parts(const uint16_t* logits, int rows, int V, int n_chunks, Top1Part* parts,
-                              cudaStream_t st) {
+void launch_reduce_fused(const uint16_t* logits, int rows, int V, int n_chunks, Top1Part* parts, int* counters,
+                         const GateBuffers& gb, int R, int k, float tau, int K, bool gate, cudaStream_t st) {
   int chunk = (V + n_chunks - 1) / n_chunks;
   chunk = (chunk + 7) / 8 * 8;
   dim3 grid(n_chunks, rows);
-  reduce_top1_parts_kernel<<<grid, 256, 0, st>>>(logits, rows, V, chunk, parts);
+  reduce_fused_kernel<<<grid, 256, 0, st>>>(logits, rows, V, chunk, n_chunks, parts, counters, gb, R, k, tau, K,
+                                            gate ? 1 : 0);
+}
+
+void launch_gate_transfer(const GateBuffers& gb, int B, int R, int k, float tau, int K, cudaStream_t st) {
+  const int warps_per_block = 4;
+  gate_transfer_kernel<<<(B + warps_per_block - 1) / warps_per_block, 32 * warps_per_block, 0, st>>>(gb, B, R, k, tau,
+                                                                                                       K);
 }
 
 void launch_combine_top1(const Top1Part* parts, int n_parts, int rows, float* conf, int32_t* argmax,
                          cudaStream_t st) {
   combine_top1_kernel<<<(rows + 7) / 8, 256, 0, st>>>(parts, n_parts, rows, conf, argmax);
-}
-
-void launch_gate_transfer(const Top1Part* parts, int n_parts, const float* conf_in, const int32_t* argmax_in,
-                          float* conf_out, int32_t* argmax_out, int32_t* prev, int32_t* persist, uint8_t* state,
-                          int32_t* tokens, int B, int R, int k, float tau, int K, uint8_t* unmask, uint8_t* accept,
-                          uint8_t* done, cudaStream_t st) {
-  const int warps_per_block = 4;
-  gate_transfer_kernel<<<(B + warps_per_block - 1) / warps_per_block, 32 * warps_per_block, 0, st>>>(
-      parts, n_parts, conf_in, argmax_in, conf_out, argmax_out, prev, persist, state, tokens, B, R, k, tau, K,
-      unmask, accept, done);
 }
 
 void launch_session_gate(const SessionGateArgs& a, cudaStream_t st) {

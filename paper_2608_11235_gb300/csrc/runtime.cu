@@ -57,6 +57,8 @@ struct DeviceCtx {
   void* scratch = nullptr;     // partials for standalone reductions
   size_t scratch_bytes = 0;
   GemmWorkspace gemm_ws{nullptr, nullptr};  // stream-K workspace for cora_op_gemm
+  int* counters = nullptr;     // completion counters of the fused reductions
+  size_t n_counters = 0;
 };
 
 std::mutex g_mu;
@@ -102,6 +104,27 @@ int scratch_reserve(DeviceCtx* c, size_t bytes, void** out) {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Partials [n_chunks, rows] (shared scratch) and n_groups completion
+// counters (a separate allocation, zeroed when grown; every launch leaves the
+// counters it used at zero).  Calls on one device are stream-ordered users of
+// the same scratch.
+int reduce_scratch(DeviceCtx* c, int n_chunks, int rows, int n_groups, Top1Part** parts, int** counters) {
+  void* p = nullptr;
+  int rc = scratch_reserve(c, size_t(n_chunks) * rows * sizeof(Top1Part), &p);
+  if (rc) return rc;
+  if (c->n_counters < size_t(n_groups)) {
+    if (c->counters) CK(cudaFree(c->counters));
+    c->counters = nullptr;
+    c->n_counters = 0;
+    CK(cudaMalloc(&c->counters, size_t(n_groups) * sizeof(int)));
+    CK(cudaMemset(c->counters, 0, size_t(n_groups) * sizeof(int)));
+    c->n_counters = size_t(n_groups);
+  }
+  *parts = static_cast<Top1Part*>(p);
+  *counters = c->counters;
+  return CORA_OK;
+}
 
 }  // namespace
 
@@ -653,8 +676,9 @@ extern "C" int cora_gate_transfer(const float* conf, const int32_t* argmax, int3
           "cora_gate_transfer: NULL pointer");
   REQUIRE(B >= 1 && R >= 1 && R <= 32, "cora_gate_transfer: need B >= 1 and 1 <= R <= 32");
   REQUIRE(k >= 0, "cora_gate_transfer: k must be >= 0");
-  launch_gate_transfer(nullptr, 0, conf, argmax, nullptr, nullptr, prev, persist, state, tokens, B, R, k, tau, K,
-                       unmask, accept, done, static_cast<cudaStream_t>(stream));
+  GateBuffers gb{const_cast<float*>(conf), const_cast<int32_t*>(argmax), prev, persist, state, tokens, unmask, accept,
+                 done};
+  launch_gate_transfer(gb, B, R, k, tau, K, static_cast<cudaStream_t>(stream));
   CK(cudaGetLastError());
   return CORA_OK;
 }
@@ -668,12 +692,12 @@ extern "C" int cora_reduce_top1(const uint16_t* logits, int32_t rows, int32_t V,
   int rc = device_ctx(&dc);
   if (rc) return rc;
   const int n = reduce_top1_parts_count(rows, V, dc->num_sms);
-  void* parts = nullptr;
-  rc = scratch_reserve(dc, size_t(n) * rows * sizeof(Top1Part), &parts);
+  Top1Part* parts = nullptr;
+  int* counters = nullptr;
+  rc = reduce_scratch(dc, n, rows, rows, &parts, &counters);
   if (rc) return rc;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  launch_reduce_top1_parts(logits, rows, V, n, static_cast<Top1Part*>(parts), st);
-  launch_combine_top1(static_cast<Top1Part*>(parts), n, rows, conf, argmax, st);
+  GateBuffers gb{conf, argmax, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+  launch_reduce_fused(logits, rows, V, n, parts, counters, gb, 1, 0, 0.f, 0, false, static_cast<cudaStream_t>(stream));
   CK(cudaGetLastError());
   return CORA_OK;
 }
@@ -690,13 +714,12 @@ extern "C" int cora_reduce_gate(const uint16_t* logits, int32_t B, int32_t R, in
   if (rc) return rc;
   const int rows = B * R;
   const int n = reduce_top1_parts_count(rows, V, dc->num_sms);
-  void* parts = nullptr;
-  rc = scratch_reserve(dc, size_t(n) * rows * sizeof(Top1Part), &parts);
+  Top1Part* parts = nullptr;
+  int* counters = nullptr;
+  rc = reduce_scratch(dc, n, rows, B, &parts, &counters);
   if (rc) return rc;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  launch_reduce_top1_parts(logits, rows, V, n, static_cast<Top1Part*>(parts), st);
-  launch_gate_transfer(static_cast<Top1Part*>(parts), n, nullptr, nullptr, conf, argmax, prev, persist, state, tokens,
-                       B, R, k, tau, K, unmask, accept, done, st);
+  GateBuffers gb{conf, argmax, prev, persist, state, tokens, unmask, accept, done};
+  launch_reduce_fused(logits, rows, V, n, parts, counters, gb, R, k, tau, K, true, static_cast<cudaStream_t>(stream));
   CK(cudaGetLastError());
   return CORA_OK;
 }

@@ -193,8 +193,13 @@ def test_reduce_top1(rows, V):
     lg = synth.gate_logits_bf16(5, 1, rows, V, hist[-1]).reshape(rows, V)
     conf = torch.empty(rows, dtype=torch.float32, device="cuda")
     arg = torch.empty(rows, dtype=torch.int32, device="cuda")
-    cora.cora_reduce_top1(dev(lg), rows, V, conf, arg)
+    lg_dev = dev(lg)
+    cora.cora_reduce_top1(lg_dev, rows, V, conf, arg)
     c_ref, a_ref = O.top1(f64(lg))
     c, a = conf.cpu().numpy(), arg.cpu().numpy()
     assert np.all(np.abs(c - c_ref) <= 1e-4 * c_ref + 1e-7)
     assert np.array_equal(a, a_ref)      # bf16 logits compare exactly on both sides; lowest id wins ties
+    conf.zero_()
+    arg.zero_()
+    cora.cora_reduce_top1(lg_dev, rows, V, conf, arg)   # second call: completion counters were left at zero
+    assert np.array_equal(conf.cpu().numpy(), c) and np.array_equal(arg.cpu().numpy(), a)
