@@ -94,8 +94,12 @@ bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64
                        uint32_t box_rows, uint32_t box_cols);
 
 int gemm_block_n(int N, int mode);
-cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K,
+cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,
                         const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st);
+bool make_gemm_out_tmap(CUtensorMap* map, void* C, int M, int ldc, int mode);
+// Generic 2-D tensor map (element size 2 = bf16, 4 = fp32), 128-byte swizzle.
+bool make_tmap_2d(CUtensorMap* map, const void* base, int elem_bytes, uint64_t rows, uint64_t cols,
+                  uint64_t row_stride_bytes, uint32_t box_rows, uint32_t box_cols);
 
 // Fused LM head + Eq. 1 partials: x [R, d] (tensor map box rows = n_pad),
 // W [V, d].  Writes parts [grid][R]; returns the number of parts used.

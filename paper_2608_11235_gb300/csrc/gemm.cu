@@ -44,7 +44,10 @@ struct GemmCfg {
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int STAGES = BN == 256 ? 4 : 6;
   static constexpr int TMEM_COLS = 2 * BN;
-  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+  // Epilogue staging: 4 warps x 2 buffers x (32 rows x 128 bytes), 128-byte
+  // swizzled, the source of the TMA stores / reductions of the outputs.
+  static constexpr int STG_BYTES = 4 * 2 * 4096;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + STG_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 };
 
 // Contiguous, even split of W iterations over G CTAs.
@@ -92,6 +95,12 @@ struct SegIter {
     ++idx;
     return true;
   }
+  // True once the segment just returned is the last one this CTA visits.
+  __device__ bool finished() const {
+    if (it1 <= it0) return true;
+    if (t_first == t_last) return idx > 0;
+    return idx >= 2 + (t_last - t_first - 1);
+  }
 };
 
 __device__ __forceinline__ void red_add_v4(float* dst, const float* a) {
@@ -121,6 +130,7 @@ struct Partials {
   const float* slots[4];  // contributors' slots, in CTA order
   int n;
   int row;                // row within the tile (0..127)
+  bool in_smem;           // slots were bulk-copied into this CTA's shared memory
 };
 
 __device__ __forceinline__ const float4* slot_chunk(const float* slot, int col, int row) {
@@ -163,7 +173,7 @@ __device__ __forceinline__ void load_acc64(uint32_t tacc, const int (&col)[4], c
     for (int q = 0; q < 4; ++q) {
       const float4* src = slot_chunk(pp.slots[p], col[q], pp.row);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) x[q][i] = __ldcg(src + i);
+      for (int i = 0; i < 4; ++i) x[q][i] = pp.in_smem ? src[i] : __ldcg(src + i);
     }
 #pragma unroll
     for (int q = 0; q < 4; ++q)
@@ -177,62 +187,157 @@ __device__ __forceinline__ void load_acc64(uint32_t tacc, const int (&col)[4], c
   }
 }
 
-// Epilogue of one 128 x BN tile for the calling thread's row, 64 columns
-// (four chunks) per step.
+// ------------------------------------------------------------ TMA epilogue
+// Each epilogue warp owns rows [32*sub, 32*sub + 32) of the tile and two
+// 4 KB staging buffers.  A "unit" is 32 rows x 128 bytes (64 bf16 or 32 fp32
+// columns): every thread writes its row into the buffer with the 128-byte
+// swizzle (16-byte chunk j of row r at chunk j ^ (r % 8): conflict-free), and
+// lane 0 hands the unit to TMA as one 2-D store (bf16 outputs) or one 2-D
+// fp32 reduce-add (the residual stream), i.e. whole 128-byte lines.
+struct Stager {
+  uint8_t* buf[2];
+  int cur;
+  int lane;
+};
+
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int c0, int c1) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1)
+               : "memory");
+}
+
+__device__ __forceinline__ void tma_reduce_add_2d(const CUtensorMap* map, const void* src, int c0, int c1) {
+  asm volatile("cp.reduce.async.bulk.tensor.2d.global.shared::cta.add.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1)
+               : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {
+  asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// Next staging buffer, once the TMA operation that last read it is done.
+__device__ __forceinline__ uint8_t* stage_acquire(Stager& sg) {
+  sg.cur ^= 1;
+  if (sg.lane == 0) bulk_wait_read<1>();
+  __syncwarp();
+  return sg.buf[sg.cur];
+}
+
+// Write 16 bytes (chunk j of this thread's row) into a swizzled unit.
+__device__ __forceinline__ void stage_chunk(uint8_t* unit, int lane, int j, uint4 v) {
+  *reinterpret_cast<uint4*>(unit + lane * 128 + ((j ^ (lane & 7)) << 4)) = v;
+}
+
+__device__ __forceinline__ void stage_bf16x16(uint8_t* unit, int lane, int j0, const float (&v)[16]) {
+  stage_chunk(unit, lane, j0, make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
+                                         pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7])));
+  stage_chunk(unit, lane, j0 + 1, make_uint4(pack_bf16x2(v[8], v[9]), pack_bf16x2(v[10], v[11]),
+                                             pack_bf16x2(v[12], v[13]), pack_bf16x2(v[14], v[15])));
+}
+
+__device__ __forceinline__ void stage_f32x16(uint8_t* unit, int lane, int j0, const float (&v)[16]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+    stage_chunk(unit, lane, j0 + q,
+                make_uint4(__float_as_uint(v[4 * q]), __float_as_uint(v[4 * q + 1]), __float_as_uint(v[4 * q + 2]),
+                           __float_as_uint(v[4 * q + 3])));
+}
+
+// Make the warp's staged unit visible to the async proxy and issue it.
+__device__ __forceinline__ void stage_issue(const Stager& sg, const CUtensorMap* map, const uint8_t* unit, int c0,
+                                            int c1, bool reduce) {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  __syncwarp();
+  if (sg.lane == 0) {
+    if (reduce)
+      tma_reduce_add_2d(map, unit, c0, c1);
+    else
+      tma_store_2d(map, unit, c0, c1);
+    bulk_commit();
+  }
+}
+
+// Epilogue of one 128 x BN tile for this warp's 32 rows (row0 = first global
+// row of the warp's box).
 template <int BN>
-__device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32_t tacc, int row, int M, int n0,
-                                                  const Partials& pp) {
-  const bool in_range = row < M;
+__device__ __forceinline__ void gemm_epilogue_warp(const GemmEpilogue& ep, const CUtensorMap* tmC, uint32_t tacc,
+                                                   int row0, int n0, const Partials& pp, Stager& sg) {
+  const int lane = sg.lane;
   if (ep.mode == CORA_EPI_STORE_BF16) {
-    uint16_t* crow = reinterpret_cast<uint16_t*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0;
 #pragma unroll 1
     for (int c = 0; c < BN; c += 64) {
       float v[4][16];
       const int cols[4] = {c, c + 16, c + 32, c + 48};
       load_acc64(tacc, cols, pp, v);
-      if (in_range)
+      uint8_t* u = stage_acquire(sg);
 #pragma unroll
-        for (int q = 0; q < 4; ++q) store_bf16x16(crow + c + 16 * q, v[q]);
+      for (int q = 0; q < 4; ++q) stage_bf16x16(u, lane, 2 * q, v[q]);
+      stage_issue(sg, tmC, u, n0 + c, row0, false);
     }
   } else if (ep.mode == CORA_EPI_RESID_F32) {
-    // h += acc as vector reductions performed at L2: no read round trip, and
-    // exactly one add per element per launch, so the result is deterministic.
-    float* crow = reinterpret_cast<float*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0;
 #pragma unroll 1
     for (int c = 0; c < BN; c += 64) {
       float v[4][16];
       const int cols[4] = {c, c + 16, c + 32, c + 48};
       load_acc64(tacc, cols, pp, v);
-      if (in_range)
-#pragma unroll
-        for (int i = 0; i < 16; ++i) red_add_v4(crow + c + 4 * i, &v[i >> 2][(i & 3) * 4]);
+      if (lane == 0) bulk_wait_read<0>();  // both buffers free
+      __syncwarp();
+      stage_f32x16(sg.buf[0], lane, 0, v[0]);
+      stage_f32x16(sg.buf[0], lane, 4, v[1]);
+      stage_f32x16(sg.buf[1], lane, 0, v[2]);
+      stage_f32x16(sg.buf[1], lane, 4, v[3]);
+      stage_issue(sg, tmC, sg.buf[0], n0 + c, row0, true);
+      stage_issue(sg, tmC, sg.buf[1], n0 + c + 32, row0, true);
+      sg.cur = 1;
     }
   } else if (ep.mode == CORA_EPI_SWIGLU) {
-    // Tile columns [0, BN/2) are gate rows, [BN/2, BN) the matching up rows
-    // of output features n0/2 .. n0/2 + BN/2.
-    uint16_t* crow = reinterpret_cast<uint16_t*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0 / 2;
+    // Tile columns [0, BN/2) are gate rows, [BN/2, BN) the matching up rows of
+    // output features n0/2 .. n0/2 + BN/2.
 #pragma unroll 1
-    for (int c = 0; c < BN / 2; c += 32) {
-      float v[4][16];
-      const int cols[4] = {c, c + 16, BN / 2 + c, BN / 2 + c + 16};
-      load_acc64(tacc, cols, pp, v);
+    for (int c = 0; c < BN / 2; c += 64) {
+      uint8_t* u = stage_acquire(sg);
+#pragma unroll 1
+      for (int h = 0; h < 64; h += 32) {
+        float v[4][16];
+        const int cols[4] = {c + h, c + h + 16, BN / 2 + c + h, BN / 2 + c + h + 16};
+        load_acc64(tacc, cols, pp, v);
 #pragma unroll
-      for (int q = 0; q < 2; ++q)
+        for (int q = 0; q < 2; ++q) {
 #pragma unroll
-        for (int j = 0; j < 16; ++j) v[q][j] = silu_f(v[q][j]) * v[q + 2][j];
-      if (in_range) {
-        store_bf16x16(crow + c, v[0]);
-        store_bf16x16(crow + c + 16, v[1]);
+          for (int j = 0; j < 16; ++j) v[q][j] = silu_f(v[q][j]) * v[q + 2][j];
+          stage_bf16x16(u, lane, (h >> 3) + 2 * q, v[q]);
+        }
       }
+      stage_issue(sg, tmC, u, n0 / 2 + c, row0, false);
     }
   } else {  // CORA_EPI_ROPE_BF16: rotate pairs (j, j + hd/2) of every head
-    uint16_t* crow = reinterpret_cast<uint16_t*>(ep.C) + static_cast<int64_t>(row) * ep.ldc + n0;
     const int hd = ep.head_dim, half = hd / 2;
-    const int pos = in_range ? row % ep.seq : 0;
+    const int pos = row0 + lane >= 0 ? (row0 + lane) % ep.seq : 0;
     const float2* tab = reinterpret_cast<const float2*>(ep.rope) + static_cast<int64_t>(pos) * half;
 #pragma unroll 1
     for (int h0 = 0; h0 < BN; h0 += hd) {
       const bool rot = n0 + h0 < ep.rope_cols;
+      // hd = 128: the two halves go to two units (both buffers); hd = 64: one unit.
+      uint8_t* u1;
+      uint8_t* u2;
+      if (hd == 128) {
+        if (lane == 0) bulk_wait_read<0>();
+        __syncwarp();
+        u1 = sg.buf[0];
+        u2 = sg.buf[1];
+        sg.cur = 1;
+      } else {
+        u1 = stage_acquire(sg);
+        u2 = u1;
+      }
 #pragma unroll 1
       for (int j0 = 0; j0 < half; j0 += 32) {
         float v[4][16];
@@ -249,15 +354,30 @@ __device__ __forceinline__ void gemm_epilogue_row(const GemmEpilogue& ep, uint32
               v[q + 2][j] = b * cs.x + a * cs.y;
             }
         }
-        if (in_range) {
-          store_bf16x16(crow + h0 + j0, v[0]);
-          store_bf16x16(crow + h0 + j0 + 16, v[1]);
-          store_bf16x16(crow + h0 + half + j0, v[2]);
-          store_bf16x16(crow + h0 + half + j0 + 16, v[3]);
-        }
+        // chunk index (16 bytes = 8 bf16) of column x within a 64-column unit
+        const int k1 = j0 >> 3;
+        const int k2 = hd == 128 ? (j0 >> 3) : ((half + j0) >> 3);
+        stage_bf16x16(u1, lane, k1, v[0]);
+        stage_bf16x16(u1, lane, k1 + 2, v[1]);
+        stage_bf16x16(u2, lane, k2, v[2]);
+        stage_bf16x16(u2, lane, k2 + 2, v[3]);
+      }
+      if (hd == 128) {
+        stage_issue(sg, tmC, u1, n0 + h0, row0, false);
+        stage_issue(sg, tmC, u2, n0 + h0 + half, row0, false);
+      } else {
+        stage_issue(sg, tmC, u1, n0 + h0, row0, false);
       }
     }
   }
+}
+
+// Contiguous global -> shared bulk copy completing `bytes` on `bar`.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
 }
 
 __device__ __forceinline__ int ld_acquire(const int* p) {
@@ -283,20 +403,24 @@ __device__ __forceinline__ bool wait_flag(const int* flag, volatile int* abort, 
 
 template <int BN>
 __global__ void __launch_bounds__(192, 1)
-    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, int M, int N,
-                   int K, GemmEpilogue ep, GemmWorkspace ws, int* err) {
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmC, int M, int N, int K, GemmEpilogue ep, GemmWorkspace ws,
+                   int* err) {
   using Cfg = GemmCfg<BN>;
   constexpr int STAGES = Cfg::STAGES;
   constexpr uint32_t IDESC = idesc_bf16_f32(kBM, BN);
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
+  uint8_t* stg = smem + STAGES * Cfg::STAGE_BYTES;  // epilogue staging (1024-aligned)
+  uint64_t* full = reinterpret_cast<uint64_t*>(stg + Cfg::STG_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  uint64_t* pbar = tempty + 2;  // completion of bulk partial copies
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint32_t pbar_phase = 0;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int num_n = N / BN;
@@ -314,12 +438,14 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(&tfull[a], 1);
       mbar_init(&tempty[a], 128);
     }
+    mbar_init(pbar, 1);
     *abort_flag = 0;
     fence_barrier_init();
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
     tma_prefetch_desc(&tmB);
+    tma_prefetch_desc(&tmC);
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
@@ -394,6 +520,11 @@ __global__ void __launch_bounds__(192, 1)
     const int sub = warp & 3;  // TMEM sub-partition this warp may access
     const int etid = threadIdx.x - 64;
     const int row_local = sub * 32 + lane;
+    Stager sg;
+    sg.buf[0] = stg + sub * 8192;
+    sg.buf[1] = stg + sub * 8192 + 4096;
+    sg.cur = 1;
+    sg.lane = lane;
     int it = 0;
     SegIter seg(blockIdx.x, G, W, KB);
     int t, kb0, kb1;
@@ -412,6 +543,7 @@ __global__ void __launch_bounds__(192, 1)
         Partials none;
         none.n = 0;
         none.row = row_local;
+        none.in_smem = false;
 #pragma unroll 1
         for (int c = 0; c < BN; c += 64) {
           float v[4][16];
@@ -435,6 +567,7 @@ __global__ void __launch_bounds__(192, 1)
       Partials pp;
       pp.n = 0;
       pp.row = row_local;
+      pp.in_smem = false;
       int c_first = 0, c_last = -1;
       if (kb1 < KB) {
         // Finisher of a split tile: contributors are the next CTAs up to the
@@ -443,17 +576,38 @@ __global__ void __launch_bounds__(192, 1)
         c_first = blockIdx.x + 1;
         c_last = c_first;
         while (c_last + 1 < G && sk_start(c_last + 1, G, W) <= last_it) ++c_last;
+        const int n_c = c_last - c_first + 1;
+        // When no segment follows, the operand ring is idle (every MMA of this
+        // CTA has completed): bulk-copy the contributors' partials into it.
+        const bool bulk = seg.finished() && n_c * kBM * BN * 4 <= STAGES * Cfg::STAGE_BYTES;
         bool fok = true;
-        if (etid == 0)
+        if (etid == 0) {
           for (int c = c_first; c <= c_last && fok; ++c) fok = wait_flag(ws.flags + c, abort_flag, err);
-        if (named_bar_or(1, 128, !fok)) break;
-        for (int c = c_first; c <= c_last; ++c) {
-          (void)ld_acquire(ws.flags + c);
-          if (pp.n < 4) pp.slots[pp.n++] = ws.partial + static_cast<int64_t>(c) * kBM * BN;
+          if (fok && bulk) {
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            const uint32_t bytes = kBM * BN * 4;
+            mbar_arrive_expect_tx(pbar, bytes * n_c);
+            for (int c = c_first; c <= c_last; ++c)
+              bulk_g2s(smem + (c - c_first) * bytes, ws.partial + static_cast<int64_t>(c) * kBM * BN, bytes, pbar);
+          }
         }
-        if (c_last - c_first + 1 > 4) record_error(err, CORA_DERR_SPLIT_WAIT);  // cannot happen: grid checked
+        if (named_bar_or(1, 128, !fok)) break;
+        if (bulk) {
+          const bool bok = mbar_wait(pbar, pbar_phase, abort_flag, err, CORA_DERR_SPLIT_WAIT);
+          pbar_phase ^= 1u;
+          if (named_bar_or(1, 128, !bok)) break;
+          pp.in_smem = true;
+          for (int c = c_first; c <= c_last && pp.n < 4; ++c)
+            pp.slots[pp.n++] = reinterpret_cast<const float*>(smem) + static_cast<int64_t>(c - c_first) * kBM * BN;
+        } else {
+          for (int c = c_first; c <= c_last; ++c) {
+            (void)ld_acquire(ws.flags + c);
+            if (pp.n < 4) pp.slots[pp.n++] = ws.partial + static_cast<int64_t>(c) * kBM * BN;
+          }
+        }
+        if (n_c > 4) record_error(err, CORA_DERR_SPLIT_WAIT);  // cannot happen: grid rule
       }
-      gemm_epilogue_row<BN>(ep, tacc, mb * kBM + row_local, M, nb * BN, pp);
+      gemm_epilogue_warp<BN>(ep, &tmC, tacc, mb * kBM + sub * 32, nb * BN, pp, sg);
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
       if (c_last >= c_first) {
@@ -462,6 +616,8 @@ __global__ void __launch_bounds__(192, 1)
           for (int c = c_first; c <= c_last; ++c) atomicExch(ws.flags + c, 0);
       }
     }
+    if (lane == 0) bulk_wait_all();  // staged outputs fully written before the CTA retires
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -490,6 +646,15 @@ static int gemm_grid(int M, int N, int K, int bn, int num_sms) {
   const int tiles = ((M + kBM - 1) / kBM) * (N / bn);
   const int KB = K / kBK;
   const long long W = static_cast<long long>(tiles) * KB;
+  if (2 * tiles <= num_sms) {
+    // Few tiles: split every tile into the same number of equal k-ranges
+    // (at most 4), so each CTA holds one piece and every finisher has its
+    // operand ring free for the partial hand-off.
+    int splits = num_sms / tiles;
+    if (splits > 4) splits = 4;
+    if (splits > KB) splits = KB;
+    return tiles * splits;
+  }
   long long g = num_sms;
   const long long max_by_share = W / ((KB + 3) / 4);
   if (g > max_by_share) g = max_by_share;
@@ -498,12 +663,12 @@ static int gemm_grid(int M, int N, int K, int bn, int num_sms) {
 }
 
 template <int BN>
-static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K,
-                                  const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms,
-                                  cudaStream_t st) {
+static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M,
+                                  int N, int K, const GemmEpilogue& ep, const GemmWorkspace& ws, int* err,
+                                  int num_sms, cudaStream_t st) {
   using Cfg = GemmCfg<BN>;
   const int grid = gemm_grid(M, N, K, BN, num_sms);
-  gemm_tc_kernel<BN><<<grid, 192, Cfg::SMEM_BYTES, st>>>(tmA, tmB, M, N, K, ep, ws, err);
+  gemm_tc_kernel<BN><<<grid, 192, Cfg::SMEM_BYTES, st>>>(tmA, tmB, tmC, M, N, K, ep, ws, err);
   return cudaGetLastError();
 }
 
@@ -515,8 +680,16 @@ cudaError_t gemm_prepare() {
                               GemmCfg<128>::SMEM_BYTES);
 }
 
-cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, const GemmEpilogue& ep,
-                        const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st) {
-  if (gemm_block_n(N, ep.mode) == 256) return launch_gemm_bn<256>(tmA, tmB, M, N, K, ep, ws, err, num_sms, st);
-  return launch_gemm_bn<128>(tmA, tmB, M, N, K, ep, ws, err, num_sms, st);
+cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,
+                        const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st) {
+  if (gemm_block_n(N, ep.mode) == 256)
+    return launch_gemm_bn<256>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);
+  return launch_gemm_bn<128>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);
+}
+
+// Output tensor map of a GEMM: 32-row x 128-byte boxes, 128-byte swizzle
+// (bf16 [M, ldc] for STORE/ROPE/SWIGLU, fp32 [M, ldc] for RESID).
+bool make_gemm_out_tmap(CUtensorMap* map, void* C, int M, int ldc, int mode) {
+  const bool f32 = mode == CORA_EPI_RESID_F32;
+  return make_tmap_2d(map, C, f32 ? 4 : 2, M, ldc, static_cast<uint64_t>(ldc) * (f32 ? 4 : 2), 32, f32 ? 32 : 64);
 }

@@ -128,17 +128,23 @@ int reduce_scratch(DeviceCtx* c, int n_chunks, int rows, int n_groups, Top1Part*
 
 }  // namespace
 
-bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
-                       uint32_t box_rows, uint32_t box_cols) {
+bool make_tmap_2d(CUtensorMap* map, const void* base, int elem_bytes, uint64_t rows, uint64_t cols,
+                  uint64_t row_stride_bytes, uint32_t box_rows, uint32_t box_cols) {
   if (!g_encode) return false;
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {row_stride_bytes};
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  CUresult r = g_encode(map, elem_bytes == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                        const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
+                       uint32_t box_rows, uint32_t box_cols) {
+  return make_tmap_2d(map, base, 2, rows, cols, row_stride_bytes, box_rows, box_cols);
 }
 
 // Sets the shared-memory attributes of every kernel instance, once per device.
@@ -327,6 +333,7 @@ struct cora_session {
   int32_t* status = nullptr;   // device {all_done (byte 0), error word}
   int32_t* status_h = nullptr; // pinned host copy
   CUtensorMap tm_xn{}, tm_attn{}, tm_act{}, tm_xf{};
+  CUtensorMap tmo_qkv{}, tmo_h{}, tmo_act{};  // GEMM output maps
   GemmWorkspace gemm_ws{nullptr, nullptr};
   cudaGraphExec_t graph = nullptr;
   int64_t batched_passes = 0;
@@ -381,19 +388,20 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr) {
     REC(CORA_KIND_RMSNORM);
     GemmEpilogue e1{s->qkv, m->n_qkv, CORA_EPI_ROPE_BF16, s->rope, s->S, c.head_dim,
                     (c.n_heads + c.n_kv_heads) * c.head_dim};
-    CK(launch_gemm(s->tm_xn, m->tm_qkv[l], M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_xn, m->tm_qkv[l], s->tmo_qkv, M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_QKV);
     launch_attention(s->qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, st);
     REC(CORA_KIND_ATTENTION);
     GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0};
-    CK(launch_gemm(s->tm_attn, m->tm_o[l], M, d, c.n_heads * c.head_dim, e2, s->gemm_ws, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_attn, m->tm_o[l], s->tmo_h, M, d, c.n_heads * c.head_dim, e2, s->gemm_ws, err, m->num_sms,
+                   st));
     REC(CORA_KIND_GEMM_O);
     launch_rmsnorm(s->h, m->ffn_norm[l], s->xn, M, d, c.norm_eps, st);
     REC(CORA_KIND_RMSNORM);
     GemmEpilogue e3{s->act, m->f_pad, CORA_EPI_SWIGLU, nullptr, 0, 0, 0};
-    CK(launch_gemm(s->tm_xn, m->tm_gu[l], M, 2 * m->f_pad, d, e3, s->gemm_ws, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_xn, m->tm_gu[l], s->tmo_act, M, 2 * m->f_pad, d, e3, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_GATE_UP);
-    CK(launch_gemm(s->tm_act, m->tm_down[l], M, d, m->f_pad, e2, s->gemm_ws, err, m->num_sms, st));
+    CK(launch_gemm(s->tm_act, m->tm_down[l], s->tmo_h, M, d, m->f_pad, e2, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_DOWN);
   }
   launch_final_norm_rows(s->h, m->final_norm, s->ctrl, s->xf, s->B, s->S, s->P, s->BL, s->n_blocks, d, c.norm_eps,
@@ -504,7 +512,10 @@ extern "C" int cora_session_create(cora_model* m, int32_t batch, const int32_t* 
   bool ok = make_tmap_bf16_2d(&s->tm_xn, s->xn, M, d, d * 2, 128, 64) &&
             make_tmap_bf16_2d(&s->tm_attn, s->attn, M, hq, hq * 2, 128, 64) &&
             make_tmap_bf16_2d(&s->tm_act, s->act, M, m->f_pad, size_t(m->f_pad) * 2, 128, 64) &&
-            make_tmap_bf16_2d(&s->tm_xf, s->xf, s->R, d, d * 2, lm_head_npad(s->R), 64);
+            make_tmap_bf16_2d(&s->tm_xf, s->xf, s->R, d, d * 2, lm_head_npad(s->R), 64) &&
+            make_gemm_out_tmap(&s->tmo_qkv, s->qkv, int(M), m->n_qkv, CORA_EPI_ROPE_BF16) &&
+            make_gemm_out_tmap(&s->tmo_h, s->h, int(M), int(d), CORA_EPI_RESID_F32) &&
+            make_gemm_out_tmap(&s->tmo_act, s->act, int(M), m->f_pad, CORA_EPI_SWIGLU);
   if (!ok) SK(fail(CORA_ECUDA, "tensor map encoding failed (session)"));
   SK(cora_session_reset(s, prompt));
   // Capture one step (every launch, then the status read-back) as a graph.
@@ -742,12 +753,13 @@ extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32
   int rc = device_ctx(&dc);
   if (rc) return rc;
   if ((rc = kernels_prepare())) return rc;
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, tc;
   const int bn = gemm_block_n(N, epilogue);
-  if (!make_tmap_bf16_2d(&ta, A, M, K, size_t(K) * 2, 128, 64) || !make_tmap_bf16_2d(&tb, B, N, K, size_t(K) * 2, bn, 64))
+  if (!make_tmap_bf16_2d(&ta, A, M, K, size_t(K) * 2, 128, 64) || !make_tmap_bf16_2d(&tb, B, N, K, size_t(K) * 2, bn, 64) ||
+      !make_gemm_out_tmap(&tc, C, M, ldc, epilogue))
     return fail(CORA_ECUDA, "cora_op_gemm: tensor map encoding failed");
   GemmEpilogue ep{C, ldc, epilogue, rope, seq, head_dim, rope_cols};
-  CK(launch_gemm(ta, tb, M, N, K, ep, dc->gemm_ws, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
+  CK(launch_gemm(ta, tb, tc, M, N, K, ep, dc->gemm_ws, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
   return CORA_OK;
 }
 
