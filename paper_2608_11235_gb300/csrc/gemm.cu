@@ -469,7 +469,10 @@ __global__ void __launch_bounds__(192, 1)
           uint8_t* sa = smem + stage * Cfg::STAGE_BYTES;
           mbar_arrive_expect_tx(&full[stage], Cfg::STAGE_BYTES);
           tma_load_2d(sa, &tmA, &full[stage], kb * kBK, mb * kBM);
-          tma_load_2d(sa + Cfg::A_BYTES, &tmB, &full[stage], kb * kBK, nb * BN);
+          // B boxes are 128 rows (the same maps feed the 2-CTA kernel's halves).
+#pragma unroll
+          for (int h = 0; h < BN / 128; ++h)
+            tma_load_2d(sa + Cfg::A_BYTES + h * 16384, &tmB, &full[stage], kb * kBK, nb * BN + h * 128);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -628,9 +631,324 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
+// ======================================================================
+// 2-CTA variant (cta_group::2): a cluster of two CTAs on two SMs computes a
+// 256 x 256 tile.  Each CTA stages its own 128 rows of A and its own 128-row
+// half of B per K step (32 KB per stage, 6 stages), so each SM moves half as
+// many operand bytes per MMA as the 1-CTA kernel; the even CTA issues
+// tcgen05.mma.cta_group::2 (M = 256, N = 256), whose result lands in both
+// CTAs' TMEM (each its own 128 rows).  Both CTAs' TMA loads complete on the
+// leader's full barrier; the leader's commits are multicast to both CTAs'
+// empty / accumulator-ready barriers; both CTAs' epilogue warps release the
+// leader's accumulator barrier.  Work split and epilogues are those of the
+// 1-CTA kernel, applied to pair-tiles (a pair is one stream-K unit; CTA
+// 2p + r owns partial slot / flag 2p + r for its 128 rows).
+// ======================================================================
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map, uint32_t bar_cluster, int c0,
+                                                 int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2 [%0], [%1, {%3, "
+      "%4}], [%2];" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma2_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive once on the barrier at this offset in both CTAs of the pair when the
+// leader's MMAs issued so far are done.
+__device__ __forceinline__ void umma2_commit_both(uint64_t* bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+          smem_u32(bar)),
+      "h"(static_cast<uint16_t>(3))
+      : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t bar_cluster) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(bar_cluster) : "memory");
+}
+
+struct Gemm2Cfg {
+  static constexpr int A_BYTES = kBM * kBK * 2;      // this CTA's 128 rows of A
+  static constexpr int B_BYTES = 128 * kBK * 2;      // this CTA's half of B
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = 6;
+  static constexpr int TMEM_COLS = 512;              // two 256-column accumulators
+  static constexpr int STG_BYTES = 4 * 2 * 4096;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + STG_BYTES + 1024 + 256;
+};
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const __grid_constant__ CUtensorMap tmC, int M, int N, int K, GemmEpilogue ep, GemmWorkspace ws,
+                    int* err) {
+  using Cfg = Gemm2Cfg;
+  constexpr int BN = 256;
+  constexpr int STAGES = Cfg::STAGES;
+  constexpr uint32_t IDESC = idesc_bf16_f32(256, BN);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* stg = smem + STAGES * Cfg::STAGE_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(stg + Cfg::STG_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* pbar = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pbar + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint32_t pbar_phase = 0;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1;
+  const int G = gridDim.x >> 1;
+  const int num_n = N / BN;
+  const int num_tiles = ((M + 255) / 256) * num_n;
+  const int KB = K / kBK;
+  const int W = num_tiles * KB;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 8);  // one arrival per epilogue warp of both CTAs
+    }
+    mbar_init(pbar, 1);
+    *abort_flag = 0;
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    tma_prefetch_desc(&tmC);
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(Cfg::TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA signal
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      SegIter seg(pair, G, W, KB);
+      int t, kb0, kb1;
+      while (seg.next(t, kb0, kb1)) {
+        const int mb = t / num_n, nb = t - mb * num_n;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err, CORA_DERR_TMA_WAIT)) goto producer_done;
+          uint8_t* sa = smem + stage * Cfg::STAGE_BYTES;
+          const uint32_t lead_full = mapa_shared(smem_u32(&full[stage]), 0);
+          if (leader) mbar_arrive_expect_tx(&full[stage], 2 * Cfg::STAGE_BYTES);
+          tma_load_2d_pair(sa, &tmA, lead_full, kb * kBK, mb * 256 + static_cast<int>(rank) * 128);
+          tma_load_2d_pair(sa + Cfg::A_BYTES, &tmB, lead_full, kb * kBK, nb * BN + static_cast<int>(rank) * 128);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+    producer_done:;
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      SegIter seg(pair, G, W, KB);
+      int t, kb0, kb1;
+      while (seg.next(t, kb0, kb1)) {
+        const int acc = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        ++it;
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1u, abort_flag, err, CORA_DERR_MMA_WAIT)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        bool ok = true;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, err, CORA_DERR_MMA_WAIT)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = smem_u32(smem + stage * Cfg::STAGE_BYTES);
+          const uint32_t b_addr = a_addr + Cfg::A_BYTES;
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k) {
+            umma2_bf16(d_tmem, sw128_kmajor_desc(a_addr + k * 32), sw128_kmajor_desc(b_addr + k * 32), IDESC,
+                       (kb > kb0 || k > 0) ? 1u : 0u);
+          }
+          umma2_commit_both(&empty[stage]);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma2_commit_both(&tfull[acc]);
+      }
+    }
+  } else {
+    const int sub = warp & 3;
+    const int etid = threadIdx.x - 64;
+    const int row_local = sub * 32 + lane;
+    const int me = 2 * pair + static_cast<int>(rank);  // this CTA's partial slot / flag
+    Stager sg;
+    sg.buf[0] = stg + sub * 8192;
+    sg.buf[1] = stg + sub * 8192 + 4096;
+    sg.cur = 1;
+    sg.lane = lane;
+    const uint32_t lead_tempty[2] = {mapa_shared(smem_u32(&tempty[0]), 0), mapa_shared(smem_u32(&tempty[1]), 0)};
+    int it = 0;
+    SegIter seg(pair, G, W, KB);
+    int t, kb0, kb1;
+    while (seg.next(t, kb0, kb1)) {
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      ++it;
+      const bool ok = mbar_wait(&tfull[acc], acc_phase, abort_flag, err, CORA_DERR_EPI_WAIT);
+      if (named_bar_or(1, 128, !ok)) break;
+      tc_fence_after();
+      const int mb = t / num_n, nb = t - mb * num_n;
+      const uint32_t tacc = tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * BN;
+      if (kb0 > 0) {
+        // Contributor: hand this CTA's 128-row partial to the tile's finisher.
+        float* slot = ws.partial + static_cast<int64_t>(me) * kBM * BN;
+        Partials none;
+        none.n = 0;
+        none.row = row_local;
+        none.in_smem = false;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 64) {
+          float v[4][16];
+          const int cols[4] = {c, c + 16, c + 32, c + 48};
+          load_acc64(tacc, cols, none, v);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            float4* dst = reinterpret_cast<float4*>(slot + (static_cast<int64_t>((c >> 4) + q) * kBM + row_local) * 16);
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+              dst[i] = make_float4(v[q][4 * i], v[q][4 * i + 1], v[q][4 * i + 2], v[q][4 * i + 3]);
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote(lead_tempty[acc]);
+        __threadfence();
+        named_bar_sync(1, 128);
+        if (etid == 0) atomicExch(ws.flags + me, 1);
+        continue;
+      }
+      Partials pp;
+      pp.n = 0;
+      pp.row = row_local;
+      pp.in_smem = false;
+      int c_first = 0, c_last = -1;
+      if (kb1 < KB) {
+        const int last_it = t * KB + KB - 1;
+        c_first = pair + 1;
+        c_last = c_first;
+        while (c_last + 1 < G && sk_start(c_last + 1, G, W) <= last_it) ++c_last;
+        const int n_c = c_last - c_first + 1;
+        const bool bulk = seg.finished() && n_c * kBM * BN * 4 <= STAGES * Cfg::STAGE_BYTES;
+        bool fok = true;
+        if (etid == 0) {
+          for (int c = c_first; c <= c_last && fok; ++c)
+            fok = wait_flag(ws.flags + 2 * c + static_cast<int>(rank), abort_flag, err);
+          if (fok && bulk) {
+            asm volatile("fence.proxy.async.global;" ::: "memory");
+            const uint32_t bytes = kBM * BN * 4;
+            mbar_arrive_expect_tx(pbar, bytes * n_c);
+            for (int c = c_first; c <= c_last; ++c)
+              bulk_g2s(smem + (c - c_first) * bytes,
+                       ws.partial + static_cast<int64_t>(2 * c + static_cast<int>(rank)) * kBM * BN, bytes, pbar);
+          }
+        }
+        if (named_bar_or(1, 128, !fok)) break;
+        if (bulk) {
+          const bool bok = mbar_wait(pbar, pbar_phase, abort_flag, err, CORA_DERR_SPLIT_WAIT);
+          pbar_phase ^= 1u;
+          if (named_bar_or(1, 128, !bok)) break;
+          pp.in_smem = true;
+          for (int c = c_first; c <= c_last && pp.n < 4; ++c)
+            pp.slots[pp.n++] = reinterpret_cast<const float*>(smem) + static_cast<int64_t>(c - c_first) * kBM * BN;
+        } else {
+          for (int c = c_first; c <= c_last; ++c) {
+            const int slot_id = 2 * c + static_cast<int>(rank);
+            (void)ld_acquire(ws.flags + slot_id);
+            if (pp.n < 4) pp.slots[pp.n++] = ws.partial + static_cast<int64_t>(slot_id) * kBM * BN;
+          }
+        }
+        if (n_c > 4) record_error(err, CORA_DERR_SPLIT_WAIT);
+      }
+      gemm_epilogue_warp<BN>(ep, &tmC, tacc, mb * 256 + static_cast<int>(rank) * 128 + sub * 32, nb * BN, pp, sg);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(lead_tempty[acc]);
+      if (c_last >= c_first) {
+        named_bar_sync(1, 128);
+        if (etid == 0)
+          for (int c = c_first; c <= c_last; ++c) atomicExch(ws.flags + 2 * c + static_cast<int>(rank), 0);
+      }
+    }
+    if (lane == 0) bulk_wait_all();
+    __syncwarp();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // no cross-CTA signal is still in flight
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(Cfg::TMEM_COLS)
+                 : "memory");
+  }
+}
+
 }  // namespace cora
 
 using namespace cora;
+
+// The 2-CTA kernel is used for M > 128 unless switched off (cora_gemm_pairs).
+static bool g_gemm_pairs_enabled = true;
+void gemm_set_pairs(bool on) { g_gemm_pairs_enabled = on; }
 
 int gemm_block_n(int N, int mode) {
   if (mode == CORA_EPI_SWIGLU) return 256;
@@ -672,9 +990,15 @@ static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB
   return cudaGetLastError();
 }
 
+// Pairs for the 2-CTA kernel: the 1-CTA rule applied to 256 x 256 pair-tiles
+// and half the SMs.
+static int gemm2_pairs(int M, int N, int K, int num_sms) { return gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2); }
+
 cudaError_t gemm_prepare() {
   cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        GemmCfg<256>::SMEM_BYTES);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(gemm_tc2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, Gemm2Cfg::SMEM_BYTES);
   if (e != cudaSuccess) return e;
   return cudaFuncSetAttribute(gemm_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               GemmCfg<128>::SMEM_BYTES);
@@ -682,6 +1006,11 @@ cudaError_t gemm_prepare() {
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,
                         const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st) {
+  if (M > 128 && N % 256 == 0 && g_gemm_pairs_enabled) {
+    const int pairs = gemm2_pairs(M, N, K, num_sms);
+    gemm_tc2_kernel<<<2 * pairs, 192, Gemm2Cfg::SMEM_BYTES, st>>>(tmA, tmB, tmC, M, N, K, ep, ws, err);
+    return cudaGetLastError();
+  }
   if (gemm_block_n(N, ep.mode) == 256)
     return launch_gemm_bn<256>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);
   return launch_gemm_bn<128>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);

@@ -280,10 +280,11 @@ extern "C" int cora_model_create(const cora_model_config* cfg, const cora_weight
     m->wgu.push_back(gu);
     m->wdown.push_back(dn);
     CUtensorMap t1, t2, t3, t4;
-    bool ok = make_tmap_bf16_2d(&t1, qkv, m->n_qkv, d, d * 2, gemm_block_n(m->n_qkv, CORA_EPI_ROPE_BF16), 64) &&
-              make_tmap_bf16_2d(&t2, wo, d, hq, hq * 2, gemm_block_n(int(d), CORA_EPI_RESID_F32), 64) &&
-              make_tmap_bf16_2d(&t3, gu, 2 * FP, d, d * 2, gemm_block_n(int(2 * FP), CORA_EPI_SWIGLU), 64) &&
-              make_tmap_bf16_2d(&t4, dn, d, FP, FP * 2, gemm_block_n(int(d), CORA_EPI_RESID_F32), 64);
+    // Weight (B operand) maps use 128-row boxes for every GEMM kernel.
+    bool ok = make_tmap_bf16_2d(&t1, qkv, m->n_qkv, d, d * 2, 128, 64) &&
+              make_tmap_bf16_2d(&t2, wo, d, hq, hq * 2, 128, 64) &&
+              make_tmap_bf16_2d(&t3, gu, 2 * FP, d, d * 2, 128, 64) &&
+              make_tmap_bf16_2d(&t4, dn, d, FP, FP * 2, 128, 64);
     if (!ok) {
       cora_model_destroy(m);
       return fail(CORA_ECUDA, "tensor map encoding failed (layer %d)", l);
@@ -754,8 +755,7 @@ extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32
   if (rc) return rc;
   if ((rc = kernels_prepare())) return rc;
   CUtensorMap ta, tb, tc;
-  const int bn = gemm_block_n(N, epilogue);
-  if (!make_tmap_bf16_2d(&ta, A, M, K, size_t(K) * 2, 128, 64) || !make_tmap_bf16_2d(&tb, B, N, K, size_t(K) * 2, bn, 64) ||
+  if (!make_tmap_bf16_2d(&ta, A, M, K, size_t(K) * 2, 128, 64) || !make_tmap_bf16_2d(&tb, B, N, K, size_t(K) * 2, 128, 64) ||
       !make_gemm_out_tmap(&tc, C, M, ldc, epilogue))
     return fail(CORA_ECUDA, "cora_op_gemm: tensor map encoding failed");
   GemmEpilogue ep{C, ldc, epilogue, rope, seq, head_dim, rope_cols};
