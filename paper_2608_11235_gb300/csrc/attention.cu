@@ -81,6 +81,8 @@ __global__ void __launch_bounds__(128) attention_kernel(const uint16_t* __restri
   const int q0 = qt * kQT;
   const int n_kt = (S + kKT - 1) / kKT;
 
+  pdl_trigger();
+  pdl_wait();
   const uint32_t sq = smem_u32(sQ);
   const uint32_t sk[2] = {smem_u32(sK0), smem_u32(sK0 + kKT * HD)};
   const uint32_t sv[2] = {smem_u32(sV0), smem_u32(sV0 + kKT * HD)};
@@ -220,9 +222,9 @@ void launch_attention(const uint16_t* qkv, uint16_t* out, int B, int S, int Hq, 
   dim3 grid((S + kQT - 1) / kQT, Hq, B);
   const int smem = (kQT + 4 * kKT) * hd * 2;
   if (hd == 128)
-    attention_kernel<128><<<grid, 128, smem, st>>>(qkv, out, S, Hq, Hkv);
+    launch_pdl(attention_kernel<128>, grid, dim3(128), smem, st, qkv, out, S, Hq, Hkv);
   else
-    attention_kernel<64><<<grid, 128, smem, st>>>(qkv, out, S, Hq, Hkv);
+    launch_pdl(attention_kernel<64>, grid, dim3(128), smem, st, qkv, out, S, Hq, Hkv);
 }
 
 cudaError_t attention_prepare() {

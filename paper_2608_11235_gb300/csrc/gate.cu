@@ -260,6 +260,8 @@ __global__ void __launch_bounds__(256) reduce_fused_kernel(const uint16_t* __res
 // block, counts the pass, and on block termination moves to the next block
 // with fresh persistence state.  Thread 0 then publishes all_done.
 __global__ void session_gate_kernel(SessionGateArgs a) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const int nw = blockDim.x >> 5;
   const int n_blocks = a.G / a.BL;
@@ -361,5 +363,5 @@ void launch_combine_top1(const Top1Part* parts, int n_parts, int rows, float* co
 void launch_session_gate(const SessionGateArgs& a, cudaStream_t st) {
   const int R = a.B * a.BL;
   const int warps = R < 32 ? R : 32;
-  session_gate_kernel<<<1, 32 * warps, 0, st>>>(a);
+  launch_pdl(session_gate_kernel, dim3(1), dim3(32 * warps), 0, st, a);
 }

@@ -455,6 +455,8 @@ __global__ void __launch_bounds__(192, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();  // A, the outputs and the workspace belong to the previous kernels
 
   if (warp == 0) {
     if (lane == 0) {
@@ -763,6 +765,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
   cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA signal
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
@@ -986,8 +990,8 @@ static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB
                                   int num_sms, cudaStream_t st) {
   using Cfg = GemmCfg<BN>;
   const int grid = gemm_grid(M, N, K, BN, num_sms);
-  gemm_tc_kernel<BN><<<grid, 192, Cfg::SMEM_BYTES, st>>>(tmA, tmB, tmC, M, N, K, ep, ws, err);
-  return cudaGetLastError();
+  return launch_pdl(gemm_tc_kernel<BN>, dim3(grid), dim3(192), Cfg::SMEM_BYTES, st, tmA, tmB, tmC, M, N, K, ep, ws,
+                    err);
 }
 
 // Pairs for the 2-CTA kernel: the 1-CTA rule applied to 256 x 256 pair-tiles
@@ -1008,8 +1012,8 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
                         const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st) {
   if (M > 128 && N % 256 == 0 && g_gemm_pairs_enabled) {
     const int pairs = gemm2_pairs(M, N, K, num_sms);
-    gemm_tc2_kernel<<<2 * pairs, 192, Gemm2Cfg::SMEM_BYTES, st>>>(tmA, tmB, tmC, M, N, K, ep, ws, err);
-    return cudaGetLastError();
+    return launch_pdl(gemm_tc2_kernel, dim3(2 * pairs), dim3(192), Gemm2Cfg::SMEM_BYTES, st, tmA, tmB, tmC, M, N, K,
+                      ep, ws, err);
   }
   if (gemm_block_n(N, ep.mode) == 256)
     return launch_gemm_bn<256>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);

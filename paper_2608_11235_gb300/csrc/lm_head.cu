@@ -80,6 +80,8 @@ __global__ void __launch_bounds__(192, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
+  pdl_wait();  // the normalised rows come from the previous kernel
 
   if (warp == 0) {
     if (lane == 0) {
@@ -223,7 +225,7 @@ template <int NPAD>
 static cudaError_t launch_head_n(const CUtensorMap& tmW, const CUtensorMap& tmX, int R, int V, int d,
                                  Top1Part* parts, int n_parts, int* err, cudaStream_t st) {
   using Cfg = HeadCfg<NPAD>;
-  lm_head_top1_kernel<NPAD><<<n_parts, 192, Cfg::SMEM_BYTES, st>>>(tmW, tmX, R, V, d, parts, err);
+  launch_pdl(lm_head_top1_kernel<NPAD>, dim3(n_parts), dim3(192), Cfg::SMEM_BYTES, st, tmW, tmX, R, V, d, parts, err);
   return cudaGetLastError();
 }
 

@@ -30,6 +30,8 @@ __global__ void synth_normal_bf16_kernel(uint16_t* __restrict__ out, int64_t cou
 // h[r, :] = float(embed[tokens[r], :]); one warp per row, 16-byte loads.
 __global__ void embed_kernel(const int32_t* __restrict__ tokens, const uint16_t* __restrict__ embed,
                              float* __restrict__ h, int M, int d) {
+  pdl_trigger();
+  pdl_wait();
   const int row = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   const int lane = threadIdx.x & 31;
   if (row >= M) return;
@@ -77,12 +79,62 @@ __device__ __forceinline__ void rmsnorm_row_warp(const float* __restrict__ x, co
   }
 }
 
-__global__ void rmsnorm_kernel(const float* __restrict__ x, const uint16_t* __restrict__ w,
-                               uint16_t* __restrict__ out, int M, int d, float eps) {
-  const int row = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-  if (row >= M) return;
-  rmsnorm_row_warp(x + static_cast<int64_t>(row) * d, w, out + static_cast<int64_t>(row) * d, d, eps,
-                   threadIdx.x & 31);
+// One 128-thread CTA per row (d <= 4096, d % 4 == 0): the row is read once
+// into registers (up to 8 float4 per thread), reduced, scaled, stored.
+constexpr int kNormThreads = 128;
+constexpr int kNormVec = 8;
+
+__device__ __forceinline__ void rmsnorm_row_cta(const float* __restrict__ x, const uint16_t* __restrict__ w,
+                                                uint16_t* __restrict__ out, int d, float eps) {
+  const float4* xv = reinterpret_cast<const float4*>(x);
+  const int nv = d >> 2;
+  float4 v[kNormVec];
+  float ss = 0.f;
+#pragma unroll
+  for (int i = 0; i < kNormVec; ++i) {
+    const int c = threadIdx.x + i * kNormThreads;
+    v[i] = c < nv ? xv[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+    ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  __shared__ float part[kNormThreads / 32];
+  if ((threadIdx.x & 31) == 0) part[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float tot = 0.f;
+#pragma unroll
+  for (int i = 0; i < kNormThreads / 32; ++i) tot += part[i];
+  const float r = rsqrtf(tot / static_cast<float>(d) + eps);
+  uint2* ov = reinterpret_cast<uint2*>(out);
+#pragma unroll
+  for (int i = 0; i < kNormVec; ++i) {
+    const int c = threadIdx.x + i * kNormThreads;
+    if (c < nv) {
+      float g0 = 1.f, g1 = 1.f, g2 = 1.f, g3 = 1.f;
+      if (w) {
+        const uint2 wv = reinterpret_cast<const uint2*>(w)[c];
+        g0 = __uint_as_float(wv.x << 16);
+        g1 = __uint_as_float(wv.x & 0xFFFF0000u);
+        g2 = __uint_as_float(wv.y << 16);
+        g3 = __uint_as_float(wv.y & 0xFFFF0000u);
+      }
+      ov[c] = make_uint2(pack_bf16x2(v[i].x * r * g0, v[i].y * r * g1), pack_bf16x2(v[i].z * r * g2, v[i].w * r * g3));
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __restrict__ x,
+                                                                const uint16_t* __restrict__ w,
+                                                                uint16_t* __restrict__ out, int M, int d, float eps) {
+  pdl_trigger();
+  pdl_wait();
+  const int row = blockIdx.x;
+  if (d <= 4 * kNormThreads * kNormVec) {
+    rmsnorm_row_cta(x + static_cast<int64_t>(row) * d, w, out + static_cast<int64_t>(row) * d, d, eps);
+  } else if (threadIdx.x < 32) {  // wider rows: one warp, two passes
+    rmsnorm_row_warp(x + static_cast<int64_t>(row) * d, w, out + static_cast<int64_t>(row) * d, d, eps,
+                     threadIdx.x & 31);
+  }
 }
 
 // Final RMSNorm on the active block's rows only: row i of sequence b is canvas
@@ -91,6 +143,8 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, const uint16_t* __re
 __global__ void final_norm_rows_kernel(const float* __restrict__ h, const uint16_t* __restrict__ w,
                                        const int32_t* __restrict__ ctrl, uint16_t* __restrict__ out, int B, int S,
                                        int P, int BL, int n_blocks, int d, float eps) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   if (r >= B * BL) return;
   const int b = r / BL, i = r % BL;
@@ -147,15 +201,16 @@ void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_
 }
 
 void launch_embed(const int32_t* tokens, const uint16_t* embed, float* h, int M, int d, cudaStream_t st) {
-  embed_kernel<<<(M + 7) / 8, 256, 0, st>>>(tokens, embed, h, M, d);
+  launch_pdl(embed_kernel, dim3((M + 7) / 8), dim3(256), 0, st, tokens, embed, h, M, d);
 }
 
 void launch_rmsnorm(const float* x, const uint16_t* w, uint16_t* out, int M, int d, float eps, cudaStream_t st) {
-  rmsnorm_kernel<<<(M + 7) / 8, 256, 0, st>>>(x, w, out, M, d, eps);
+  launch_pdl(rmsnorm_kernel, dim3(M), dim3(kNormThreads), 0, st, x, w, out, M, d, eps);
 }
 
 void launch_final_norm_rows(const float* h, const uint16_t* w, const int32_t* ctrl, uint16_t* out, int B, int S,
                             int P, int BL, int n_blocks, int d, float eps, cudaStream_t st) {
   const int R = B * BL;
-  final_norm_rows_kernel<<<(R + 7) / 8, 256, 0, st>>>(h, w, ctrl, out, B, S, P, BL, n_blocks, d, eps);
+  launch_pdl(final_norm_rows_kernel, dim3((R + 7) / 8), dim3(256), 0, st, h, w, ctrl, out, B, S, P, BL, n_blocks, d,
+             eps);
 }
