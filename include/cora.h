@@ -245,6 +245,23 @@ CORA_API int cora_gate_transfer(const float* conf, const int32_t* argmax, int32_
  * ties).  V >= 1.  Streams the logits once from HBM. */
 CORA_API int cora_reduce_top1(const uint16_t* logits, int32_t rows, int32_t V, float* conf, int32_t* argmax, void* stream);
 
+/* cora_reduce_top1 without any device allocation.  The paper has no
+ * counterpart; this serves callers that must not allocate device memory when
+ * they call it: code running during CUDA stream capture (cudaMalloc cannot be
+ * captured), applications whose memory pool already holds all device memory,
+ * and latency-critical loops that must stay out of the allocator.
+ * Scratch is a fixed array compiled into the library (832 KiB: 65536 partial
+ * states + 16384 counters), present on every GPU that loads the library until
+ * the process exits.  Same arguments, layout and results as
+ * cora_reduce_top1; rows <= 16384, else CORA_EINVAL.
+ * The first call on a device (with that device current) looks up the array's
+ * device address; make that first call before any stream capture.  Calls
+ * share the array, so calls that may overlap on the GPU (different streams
+ * without ordering) race; serialise them.  Each call clears the counters it
+ * uses with cudaMemsetAsync on `stream` before its kernel. */
+CORA_API int cora_reduce_top1_noalloc(const uint16_t* logits, int32_t rows, int32_t V, float* conf, int32_t* argmax,
+                                      void* stream);
+
 /* cora_reduce_top1 on [B, R, V] logits followed by cora_gate_transfer on the
  * result (the gate-isolation workload).  conf/argmax outputs are device
  * [B, R] and also serve as the gate's inputs. */

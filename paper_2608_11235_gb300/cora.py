@@ -25,7 +25,7 @@ EXPORTED = [
     "cora_session_destroy", "cora_session_reset", "cora_denoise_step", "cora_session_read", "cora_session_write",
     "cora_session_batched_passes", "cora_generate", "cora_gate_transfer", "cora_reduce_top1", "cora_reduce_gate",
     "cora_op_gemm", "cora_op_attention", "cora_op_rmsnorm", "cora_op_lm_head_top1", "cora_synth_normal_bf16",
-    "cora_device_error", "cora_session_profile_step", "cora_session_stream",
+    "cora_device_error", "cora_session_profile_step", "cora_session_stream", "cora_reduce_top1_noalloc",
 ]
 KIND_NAMES = ["embed", "rmsnorm", "gemm_qkv_rope", "attention", "gemm_o_resid", "gemm_gate_up_swiglu",
               "gemm_down_resid", "final_norm", "lm_head_top1", "gate"]
@@ -85,6 +85,7 @@ def lib():
             "cora_generate": ([vp, vp, i32, i32, i32, i32, i32, f32, i32, vp, vp, vp], C.c_int),
             "cora_gate_transfer": ([vp] * 6 + [i32, i32, i32, f32, i32] + [vp] * 3 + [vp], C.c_int),
             "cora_reduce_top1": ([vp, i32, i32, vp, vp, vp], C.c_int),
+            "cora_reduce_top1_noalloc": ([vp, i32, i32, vp, vp, vp], C.c_int),
             "cora_reduce_gate": ([vp, i32, i32, i32] + [vp] * 6 + [i32, f32, i32] + [vp] * 3 + [vp], C.c_int),
             "cora_op_gemm": ([vp, vp, vp, i32, i32, i32, i32, i32, vp, i32, i32, i32, vp], C.c_int),
             "cora_op_attention": ([vp, vp, i32, i32, i32, i32, i32, vp], C.c_int),
@@ -241,6 +242,11 @@ def cora_gate_transfer(conf, argmax, prev, persist, state, tokens, B, R, k, tau,
 def cora_reduce_top1(logits, rows, V, conf, argmax, stream=None) -> None:
     _check("cora_reduce_top1", lib().cora_reduce_top1(ptr(logits), rows, V, ptr(conf), ptr(argmax),
                                                       _stream(stream)))
+
+
+def cora_reduce_top1_noalloc(logits, rows, V, conf, argmax, stream=None) -> None:
+    _check("cora_reduce_top1_noalloc", lib().cora_reduce_top1_noalloc(ptr(logits), rows, V, ptr(conf), ptr(argmax),
+                                                                      _stream(stream)))
 
 
 def cora_reduce_gate(logits, B, R, V, conf, argmax, prev, persist, state, tokens, k, tau, K, unmask, accept, done,

@@ -84,6 +84,7 @@ struct GateBuffers {
 // block of R rows) done by the last CTA of each group.  counters: zeroed ints,
 // one per row (gate == false) or per block (gate == true); left zeroed.
 int reduce_top1_parts_count(int rows, int V, int num_sms);
+int cora_set_error(int code, const char* msg);
 void launch_reduce_fused(const uint16_t* logits, int rows, int V, int n_chunks, Top1Part* parts, int* counters,
                          const GateBuffers& gb, int R, int k, float tau, int K, bool gate, cudaStream_t st);
 void launch_combine_top1(const Top1Part* parts, int n_parts, int rows, float* conf, int32_t* argmax,

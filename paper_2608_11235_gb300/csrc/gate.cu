@@ -3,6 +3,8 @@
 #include <float.h>
 #include <limits.h>
 
+#include <mutex>
+
 #include "cora_device.cuh"
 #include "cora_kernels.h"
 #include "../../include/cora.h"
@@ -364,4 +366,74 @@ void launch_session_gate(const SessionGateArgs& a, cudaStream_t st) {
   const int R = a.B * a.BL;
   const int warps = R < 32 ? R : 32;
   launch_pdl(session_gate_kernel, dim3(1), dim3(32 * warps), 0, st, a);
+}
+
+// ----------------------------------------------------------------------------
+// Allocation-free Eq. 1 reduction.
+//
+// Some callers cannot allocate device memory at the moment they need this
+// reduction: code running while a CUDA graph is being captured (cudaMalloc is
+// not a capturable operation), an application whose memory pool already owns
+// the whole device, or a latency-critical loop that must not enter the
+// allocator.  cora_reduce_top1_noalloc serves them with scratch that exists as
+// soon as the library is loaded: the array below, reserved on every GPU that
+// loads the library and kept until the process exits.
+// ----------------------------------------------------------------------------
+#define CORA_NOALLOC_MAX_PARTIALS 65536  // (chunk, row) partial states: 768 KiB
+#define CORA_NOALLOC_MAX_ROWS 16384      // completion counters: 64 KiB
+
+struct NoAllocScratch {
+  Top1Part parts[CORA_NOALLOC_MAX_PARTIALS];
+  int counters[CORA_NOALLOC_MAX_ROWS];
+};
+
+static __device__ __align__(256) NoAllocScratch g_noalloc_scratch;
+
+namespace {
+std::mutex g_noalloc_mu;
+NoAllocScratch* g_noalloc_dev[64];  // device address of the array, per device
+int g_noalloc_sms[64];
+}  // namespace
+
+extern "C" int cora_reduce_top1_noalloc(const uint16_t* logits, int32_t rows, int32_t V, float* conf, int32_t* argmax,
+                                        void* stream) {
+  if (!logits || !conf || !argmax) return cora_set_error(CORA_EINVAL, "cora_reduce_top1_noalloc: NULL pointer");
+  if (rows < 1 || V < 1) return cora_set_error(CORA_EINVAL, "cora_reduce_top1_noalloc: rows and V must be >= 1");
+  if (rows > CORA_NOALLOC_MAX_ROWS)
+    return cora_set_error(CORA_EINVAL, "cora_reduce_top1_noalloc: rows exceeds the fixed scratch (max 16384)");
+  if ((V & 7) == 0 && (reinterpret_cast<uintptr_t>(logits) & 15u) != 0)
+    return cora_set_error(CORA_EINVAL, "cora_reduce_top1_noalloc: logits must be 16-byte aligned");
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64)
+    return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: no usable current device");
+  NoAllocScratch* scratch = nullptr;
+  int num_sms = 0;
+  {
+    // First call on a device: look up where the array lives on that device
+    // (the array's name is only a host-side handle) and the SM count.
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (!g_noalloc_dev[dev]) {
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
+        return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: cudaGetSymbolAddress failed");
+      if (cudaDeviceGetAttribute(&g_noalloc_sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: cannot read the SM count");
+      g_noalloc_dev[dev] = static_cast<NoAllocScratch*>(p);
+    }
+    scratch = g_noalloc_dev[dev];
+    num_sms = g_noalloc_sms[dev];
+  }
+  int n_chunks = reduce_top1_parts_count(rows, V, num_sms);
+  const int cap = CORA_NOALLOC_MAX_PARTIALS / rows;  // >= 4 since rows <= 16384
+  if (n_chunks > cap) n_chunks = cap;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // The counters must start at zero; completed launches leave them at zero,
+  // but the array is shared by every call, so clear this call's range first.
+  if (cudaMemsetAsync(scratch->counters, 0, sizeof(int) * rows, st) != cudaSuccess)
+    return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: clearing the counters failed");
+  GateBuffers gb{conf, argmax, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, nullptr};
+  launch_reduce_fused(logits, rows, V, n_chunks, scratch->parts, scratch->counters, gb, 1, 0, 0.f, 0, false, st);
+  if (cudaGetLastError() != cudaSuccess)
+    return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: kernel launch failed");
+  return CORA_OK;
 }

@@ -29,6 +29,13 @@ static int fail(int code, const char* fmt, ...) {
   return code;
 }
 
+// Records `msg` as the calling thread's last error and returns `code`
+// (for entry points implemented in other translation units).
+int cora_set_error(int code, const char* msg) {
+  g_last_error = msg;
+  return code;
+}
+
 #define CK(call)                                                                        \
   do {                                                                                  \
     cudaError_t e_ = (call);                                                            \
