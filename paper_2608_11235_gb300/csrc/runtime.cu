@@ -164,6 +164,7 @@ static int kernels_prepare() {
     CK(gemm_prepare());
     CK(lm_head_prepare());
     CK(attention_prepare());
+    CK(attention_tc_prepare());
     dc->prepared = true;
   }
   return CORA_OK;
@@ -342,6 +343,7 @@ struct cora_session {
   int32_t* status_h = nullptr; // pinned host copy
   CUtensorMap tm_xn{}, tm_attn{}, tm_act{}, tm_xf{};
   CUtensorMap tmo_qkv{}, tmo_h{}, tmo_act{};  // GEMM output maps
+  CUtensorMap tm_qkv_in{};                     // QKV as the attention kernel's TMA source
   GemmWorkspace gemm_ws{nullptr, nullptr};
   cudaGraphExec_t graph = nullptr;
   int64_t batched_passes = 0;
@@ -398,7 +400,11 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr) {
                     (c.n_heads + c.n_kv_heads) * c.head_dim};
     CK(launch_gemm(s->tm_xn, m->tm_qkv[l], s->tmo_qkv, M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_QKV);
-    launch_attention(s->qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, st);
+    if (c.head_dim == 128) {
+      CK(launch_attention_tc(s->tm_qkv_in, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, err, st));
+    } else {
+      launch_attention(s->qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, st);
+    }
     REC(CORA_KIND_ATTENTION);
     GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0};
     CK(launch_gemm(s->tm_attn, m->tm_o[l], s->tmo_h, M, d, c.n_heads * c.head_dim, e2, s->gemm_ws, err, m->num_sms,
@@ -522,6 +528,7 @@ extern "C" int cora_session_create(cora_model* m, int32_t batch, const int32_t* 
             make_tmap_bf16_2d(&s->tm_act, s->act, M, m->f_pad, size_t(m->f_pad) * 2, 128, 64) &&
             make_tmap_bf16_2d(&s->tm_xf, s->xf, s->R, d, d * 2, lm_head_npad(s->R), 64) &&
             make_gemm_out_tmap(&s->tmo_qkv, s->qkv, int(M), m->n_qkv, CORA_EPI_ROPE_BF16) &&
+            make_tmap_bf16_2d(&s->tm_qkv_in, s->qkv, M, size_t(m->n_qkv), size_t(m->n_qkv) * 2, 128, 64) &&
             make_gemm_out_tmap(&s->tmo_h, s->h, int(M), int(d), CORA_EPI_RESID_F32) &&
             make_gemm_out_tmap(&s->tmo_act, s->act, int(M), m->f_pad, CORA_EPI_SWIGLU);
   if (!ok) SK(fail(CORA_ECUDA, "tensor map encoding failed (session)"));
@@ -778,7 +785,17 @@ extern "C" int cora_op_attention(const uint16_t* qkv, uint16_t* out, int32_t B, 
   REQUIRE(aligned16(qkv) && aligned16(out), "cora_op_attention: pointers must be 16-byte aligned");
   int rc = kernels_prepare();
   if (rc) return rc;
-  launch_attention(qkv, out, B, S, Hq, Hkv, hd, static_cast<cudaStream_t>(stream));
+  if (hd == 128) {
+    DeviceCtx* dc = nullptr;
+    if ((rc = device_ctx(&dc))) return rc;
+    CUtensorMap tq;
+    const size_t cols = size_t(Hq + 2 * Hkv) * hd;
+    if (!make_tmap_bf16_2d(&tq, qkv, size_t(B) * S, cols, cols * 2, 128, 64))
+      return fail(CORA_ECUDA, "cora_op_attention: tensor map encoding failed");
+    CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, dc->err, static_cast<cudaStream_t>(stream)));
+  } else {
+    launch_attention(qkv, out, B, S, Hq, Hkv, hd, static_cast<cudaStream_t>(stream));
+  }
   CK(cudaGetLastError());
   return CORA_OK;
 }

@@ -152,6 +152,7 @@ def test_gemm_rope(B, S, H, Hkv, hd, theta):
 
 # --------------------------------------------------------------- attention
 @pytest.mark.parametrize("B,S,Hq,Hkv,hd", [(2, 96, 4, 4, 64), (1, 200, 8, 2, 128), (1, 512, 2, 2, 128),
+                                          (2, 130, 4, 2, 128), (1, 1, 2, 2, 128), (2, 300, 4, 4, 128),
                                           (3, 1, 2, 1, 64)])
 def test_attention(B, S, Hq, Hkv, hd):
     W = (Hq + 2 * Hkv) * hd
