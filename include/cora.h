@@ -247,9 +247,10 @@ CORA_API int cora_reduce_top1(const uint16_t* logits, int32_t rows, int32_t V, f
 
 /* cora_reduce_top1 without any device allocation.  The paper has no
  * counterpart; this serves callers that must not allocate device memory when
- * they call it: code running during CUDA stream capture (cudaMalloc cannot be
- * captured), applications whose memory pool already holds all device memory,
- * and latency-critical loops that must stay out of the allocator.
+ * they call it: applications whose memory pool already holds all device
+ * memory (a cudaMalloc would fail or evict their cache), and latency-critical
+ * loops that must stay out of the allocator (cudaMalloc and cudaFree
+ * synchronise the device).
  * Scratch is a fixed array compiled into the library (832 KiB: 65536 partial
  * states + 16384 counters), present on every GPU that loads the library until
  * the process exits.  Same arguments, layout and results as

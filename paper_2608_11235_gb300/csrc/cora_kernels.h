@@ -101,6 +101,14 @@ struct GemmEpilogue {
   int seq;
   int head_dim;
   int rope_cols;
+  // 1 when B is not written by any kernel that may still run on the stream
+  // (model weights): the 2-CTA kernel then starts loading B before waiting
+  // for the previous kernel (programmatic dependent launch).
+  int b_static;
+  // Set by launch_gemm: equal k-splits per tile (0 = stream-K) and their
+  // skew toward the finishing piece, in k-blocks.
+  int splits;
+  int split_skew;
 };
 
 // Stream-K workspace: one fp32 partial slot of 128 x 256 per CTA plus one

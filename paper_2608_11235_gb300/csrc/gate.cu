@@ -372,10 +372,10 @@ void launch_session_gate(const SessionGateArgs& a, cudaStream_t st) {
 // Allocation-free Eq. 1 reduction.
 //
 // Some callers cannot allocate device memory at the moment they need this
-// reduction: code running while a CUDA graph is being captured (cudaMalloc is
-// not a capturable operation), an application whose memory pool already owns
-// the whole device, or a latency-critical loop that must not enter the
-// allocator.  cora_reduce_top1_noalloc serves them with scratch that exists as
+// reduction: an application whose memory pool already owns the whole device
+// (a cudaMalloc would fail or force it to give memory back), or a
+// latency-critical loop that must not enter the allocator (cudaMalloc and
+// cudaFree synchronise the device).  cora_reduce_top1_noalloc serves them with scratch that exists as
 // soon as the library is loaded: the array below, reserved on every GPU that
 // loads the library and kept until the process exits.
 // ----------------------------------------------------------------------------

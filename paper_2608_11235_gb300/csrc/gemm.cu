@@ -50,10 +50,22 @@ struct GemmCfg {
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + STG_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 };
 
-// Contiguous, even split of W iterations over G CTAs.
-__device__ __forceinline__ int sk_start(int c, int G, int W) {
-  return static_cast<int>((static_cast<long long>(c) * W) / G);
-}
+// Division of the W = tiles * KB (tile, k-block) iterations among G CTAs
+// (or CTA pairs).  Uniform (stream-K): unit c starts at c W / G.  Skewed
+// equal splits (G = tiles * S): the piece holding k-block 0, which finishes
+// the tile, is skew * (S - 1) k-blocks longer than KB / S and every other
+// piece skew shorter, so the other pieces' partials are written while the
+// finisher is still issuing MMAs instead of after.
+struct WorkSplit {
+  int G, W, KB, S, skew;
+  __device__ int start(int c) const {
+    if (skew > 0) {
+      const int t = c / S, s = c - t * S;
+      return t * KB + (s == 0 ? 0 : KB - (S - s) * (KB / S - skew));
+    }
+    return static_cast<int>((static_cast<long long>(c) * W) / G);
+  }
+};
 
 // A CTA's iteration range as segments (tile, kb0, kb1), visited in the order
 // (1) its first segment (a contributor when it starts mid-tile), (2) its
@@ -62,10 +74,10 @@ __device__ __forceinline__ int sk_start(int c, int G, int W) {
 // hand-off and fix-up overlap the MMAs of the whole tiles.
 struct SegIter {
   int it0, it1, kb_per_tile, t_first, t_last, idx;
-  __device__ SegIter(int c, int G, int W, int KB)
-      : it0(sk_start(c, G, W)), it1(sk_start(c + 1, G, W)), kb_per_tile(KB), idx(0) {
-    t_first = it0 / KB;
-    t_last = it1 > it0 ? (it1 - 1) / KB : t_first - 1;
+  __device__ SegIter(int c, const WorkSplit& ws)
+      : it0(ws.start(c)), it1(ws.start(c + 1)), kb_per_tile(ws.KB), idx(0) {
+    t_first = it0 / ws.KB;
+    t_last = it1 > it0 ? (it1 - 1) / ws.KB : t_first - 1;
   }
   __device__ bool next(int& t, int& kb0, int& kb1) {
     if (it1 <= it0) return false;
@@ -103,6 +115,26 @@ struct SegIter {
   }
 };
 
+// Walks a CTA's (tile, k-block) sequence in the order the producer loads it.
+struct KbCursor {
+  SegIter seg;
+  int t, kb, kb1;
+  bool valid;
+  __device__ KbCursor(int c, const WorkSplit& ws) : seg(c, ws) {
+    int kb0 = 0;
+    valid = seg.next(t, kb0, kb1);
+    kb = kb0;
+  }
+  __device__ void advance() {
+    if (!valid) return;
+    if (++kb >= kb1) {
+      int kb0 = 0;
+      valid = seg.next(t, kb0, kb1);
+      kb = kb0;
+    }
+  }
+};
+
 __device__ __forceinline__ void red_add_v4(float* dst, const float* a) {
   asm volatile("red.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(dst), "f"(a[0]), "f"(a[1]), "f"(a[2]), "f"(a[3])
                : "memory");
@@ -124,8 +156,11 @@ __device__ __forceinline__ void store_bf16x16(uint16_t* dst, const float (&v)[16
   reinterpret_cast<uint4*>(dst)[1] = b;
 }
 
-// Partial accumulators of split tiles: slot per CTA, [BN/16][128 rows][16]
-// fp32, so a warp's 16-column chunk is 2 KB contiguous.
+// Partial accumulators of split tiles: slot per CTA, [BN/16][4][128 rows][4]
+// fp32.  Thread r owns row r; its float4 i of 16-column chunk q sits at
+// index (4 q + i) * 128 + r, so one warp-wide float4 access covers 512
+// contiguous bytes (whole 128-byte lines in global memory, no bank conflicts
+// in shared memory).
 struct Partials {
   const float* slots[4];  // contributors' slots, in CTA order
   int n;
@@ -133,9 +168,7 @@ struct Partials {
   bool in_smem;           // slots were bulk-copied into this CTA's shared memory
 };
 
-__device__ __forceinline__ const float4* slot_chunk(const float* slot, int col, int row) {
-  return reinterpret_cast<const float4*>(slot + (static_cast<int64_t>(col >> 4) * kBM + row) * 16);
-}
+__device__ __forceinline__ int part_f4(int col, int i, int row) { return ((col >> 4) * 4 + i) * kBM + row; }
 
 // Loads four 16-column accumulator chunks (columns col[0..3]) under one TMEM
 // wait, then adds every contributor's partial; all global loads of one
@@ -171,9 +204,12 @@ __device__ __forceinline__ void load_acc64(uint32_t tacc, const int (&col)[4], c
     float4 x[4][4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      const float4* src = slot_chunk(pp.slots[p], col[q], pp.row);
+      const float4* src = reinterpret_cast<const float4*>(pp.slots[p]);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) x[q][i] = pp.in_smem ? src[i] : __ldcg(src + i);
+      for (int i = 0; i < 4; ++i) {
+        const int o = part_f4(col[q], i, pp.row);
+        x[q][i] = pp.in_smem ? src[o] : __ldcg(src + o);
+      }
     }
 #pragma unroll
     for (int q = 0; q < 4; ++q)
@@ -428,6 +464,7 @@ __global__ void __launch_bounds__(192, 1)
   const int KB = K / kBK;
   const int W = num_tiles * KB;
   const int G = gridDim.x;
+  const WorkSplit wsplit{G, W, KB, ep.splits, ep.split_skew};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -462,7 +499,7 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      SegIter seg(blockIdx.x, G, W, KB);
+      SegIter seg(blockIdx.x, wsplit);
       int t, kb0, kb1;
       while (seg.next(t, kb0, kb1)) {
         const int mb = t / num_n, nb = t - mb * num_n;
@@ -488,7 +525,7 @@ __global__ void __launch_bounds__(192, 1)
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
-      SegIter seg(blockIdx.x, G, W, KB);
+      SegIter seg(blockIdx.x, wsplit);
       int t, kb0, kb1;
       while (seg.next(t, kb0, kb1)) {
         const int acc = it & 1;
@@ -531,7 +568,7 @@ __global__ void __launch_bounds__(192, 1)
     sg.cur = 1;
     sg.lane = lane;
     int it = 0;
-    SegIter seg(blockIdx.x, G, W, KB);
+    SegIter seg(blockIdx.x, wsplit);
     int t, kb0, kb1;
     while (seg.next(t, kb0, kb1)) {
       const int acc = it & 1;
@@ -556,10 +593,11 @@ __global__ void __launch_bounds__(192, 1)
           load_acc64(tacc, cols, none, v);
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
-            float4* dst = reinterpret_cast<float4*>(slot + (static_cast<int64_t>((c >> 4) + q) * kBM + row_local) * 16);
+            float4* dst = reinterpret_cast<float4*>(slot);
 #pragma unroll
             for (int i = 0; i < 4; ++i)
-              dst[i] = make_float4(v[q][4 * i], v[q][4 * i + 1], v[q][4 * i + 2], v[q][4 * i + 3]);
+              dst[part_f4(c + 16 * q, i, row_local)] =
+                  make_float4(v[q][4 * i], v[q][4 * i + 1], v[q][4 * i + 2], v[q][4 * i + 3]);
           }
         }
         tc_fence_before();
@@ -580,7 +618,7 @@ __global__ void __launch_bounds__(192, 1)
         const int last_it = t * KB + KB - 1;
         c_first = blockIdx.x + 1;
         c_last = c_first;
-        while (c_last + 1 < G && sk_start(c_last + 1, G, W) <= last_it) ++c_last;
+        while (c_last + 1 < G && wsplit.start(c_last + 1) <= last_it) ++c_last;
         const int n_c = c_last - c_first + 1;
         // When no segment follows, the operand ring is idle (every MMA of this
         // CTA has completed): bulk-copy the contributors' partials into it.
@@ -735,6 +773,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
   const int num_tiles = ((M + 255) / 256) * num_n;
   const int KB = K / kBK;
   const int W = num_tiles * KB;
+  const WorkSplit wsplit{G, W, KB, ep.splits, ep.split_skew};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -766,23 +805,39 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   pdl_trigger();
+
+  // With ep.b_static, the ring's first B tiles are loaded before waiting for
+  // the previous kernel: B (the weights) does not depend on it, A does.
+  const int b_row = static_cast<int>(rank) * 128;
+  int n_pre = 0, n_issued = 0;
+  if (warp == 0 && lane == 0 && ep.b_static) {
+    for (KbCursor cur(pair, wsplit); n_pre < STAGES && cur.valid; ++n_pre, cur.advance()) {
+      uint8_t* sa = smem + n_pre * Cfg::STAGE_BYTES;
+      if (leader) mbar_arrive_expect_tx(&full[n_pre], 2 * Cfg::STAGE_BYTES);
+      tma_load_2d_pair(sa + Cfg::A_BYTES, &tmB, mapa_shared(smem_u32(&full[n_pre]), 0), cur.kb * kBK,
+                       (cur.t % num_n) * BN + b_row);
+    }
+  }
   pdl_wait();
 
   if (warp == 0) {
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
-      SegIter seg(pair, G, W, KB);
+      SegIter seg(pair, wsplit);
       int t, kb0, kb1;
       while (seg.next(t, kb0, kb1)) {
         const int mb = t / num_n, nb = t - mb * num_n;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err, CORA_DERR_TMA_WAIT)) goto producer_done;
           uint8_t* sa = smem + stage * Cfg::STAGE_BYTES;
           const uint32_t lead_full = mapa_shared(smem_u32(&full[stage]), 0);
-          if (leader) mbar_arrive_expect_tx(&full[stage], 2 * Cfg::STAGE_BYTES);
+          if (n_issued >= n_pre) {  // (the first n_pre slots are free and already expect their bytes)
+            if (!mbar_wait(&empty[stage], phase ^ 1u, abort_flag, err, CORA_DERR_TMA_WAIT)) goto producer_done;
+            if (leader) mbar_arrive_expect_tx(&full[stage], 2 * Cfg::STAGE_BYTES);
+            tma_load_2d_pair(sa + Cfg::A_BYTES, &tmB, lead_full, kb * kBK, nb * BN + b_row);
+          }
           tma_load_2d_pair(sa, &tmA, lead_full, kb * kBK, mb * 256 + static_cast<int>(rank) * 128);
-          tma_load_2d_pair(sa + Cfg::A_BYTES, &tmB, lead_full, kb * kBK, nb * BN + static_cast<int>(rank) * 128);
+          ++n_issued;
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -796,7 +851,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
-      SegIter seg(pair, G, W, KB);
+      SegIter seg(pair, wsplit);
       int t, kb0, kb1;
       while (seg.next(t, kb0, kb1)) {
         const int acc = it & 1;
@@ -841,7 +896,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
     sg.lane = lane;
     const uint32_t lead_tempty[2] = {mapa_shared(smem_u32(&tempty[0]), 0), mapa_shared(smem_u32(&tempty[1]), 0)};
     int it = 0;
-    SegIter seg(pair, G, W, KB);
+    SegIter seg(pair, wsplit);
     int t, kb0, kb1;
     while (seg.next(t, kb0, kb1)) {
       const int acc = it & 1;
@@ -866,10 +921,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
           load_acc64(tacc, cols, none, v);
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
-            float4* dst = reinterpret_cast<float4*>(slot + (static_cast<int64_t>((c >> 4) + q) * kBM + row_local) * 16);
+            float4* dst = reinterpret_cast<float4*>(slot);
 #pragma unroll
             for (int i = 0; i < 4; ++i)
-              dst[i] = make_float4(v[q][4 * i], v[q][4 * i + 1], v[q][4 * i + 2], v[q][4 * i + 3]);
+              dst[part_f4(c + 16 * q, i, row_local)] =
+                  make_float4(v[q][4 * i], v[q][4 * i + 1], v[q][4 * i + 2], v[q][4 * i + 3]);
           }
         }
         tc_fence_before();
@@ -889,7 +945,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
         const int last_it = t * KB + KB - 1;
         c_first = pair + 1;
         c_last = c_first;
-        while (c_last + 1 < G && sk_start(c_last + 1, G, W) <= last_it) ++c_last;
+        while (c_last + 1 < G && wsplit.start(c_last + 1) <= last_it) ++c_last;
         const int n_c = c_last - c_first + 1;
         const bool bulk = seg.finished() && n_c * kBM * BN * 4 <= STAGES * Cfg::STAGE_BYTES;
         bool fok = true;
@@ -961,20 +1017,34 @@ int gemm_block_n(int N, int mode) {
 
 size_t gemm_workspace_bytes(int num_sms) { return static_cast<size_t>(num_sms) * kBM * 256 * sizeof(float); }
 
+// A contributor's partial hand-off (epilogue stores, fence, flag) takes about
+// as long as 13 k-block MMA steps; skewed equal splits hide it behind the
+// finisher's extra k-blocks (skew * S >= 13).
+constexpr int kSkewTotal = 14;
+
 // Grid for a stream-K launch: one CTA per SM, but every CTA gets at least
 // ceil(KB/4) iterations, so a split tile has at most four contributors
-// besides its finisher; never more CTAs than iterations.
-static int gemm_grid(int M, int N, int K, int bn, int num_sms) {
+// besides its finisher; never more CTAs than iterations.  Sets the split
+// fields of `ep` (uniform unless equal splits apply).
+static int gemm_grid(int M, int N, int K, int bn, int num_sms, GemmEpilogue& ep) {
   const int tiles = ((M + kBM - 1) / kBM) * (N / bn);
   const int KB = K / kBK;
   const long long W = static_cast<long long>(tiles) * KB;
+  ep.splits = 0;
+  ep.split_skew = 0;
   if (2 * tiles <= num_sms) {
-    // Few tiles: split every tile into the same number of equal k-ranges
-    // (at most 4), so each CTA holds one piece and every finisher has its
-    // operand ring free for the partial hand-off.
+    // Few tiles: split every tile into the same number of k-ranges (at most
+    // 4), so each CTA holds one piece and every finisher has its operand
+    // ring free for the partial hand-off; skewed toward the finisher.
     int splits = num_sms / tiles;
     if (splits > 4) splits = 4;
     if (splits > KB) splits = KB;
+    if (splits >= 2 && KB % splits == 0) {
+      int skew = (kSkewTotal + splits - 1) / splits;
+      if (skew > KB / (2 * splits)) skew = KB / (2 * splits);
+      ep.splits = splits;
+      ep.split_skew = skew;
+    }
     return tiles * splits;
   }
   long long g = num_sms;
@@ -989,14 +1059,17 @@ static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB
                                   int N, int K, const GemmEpilogue& ep, const GemmWorkspace& ws, int* err,
                                   int num_sms, cudaStream_t st) {
   using Cfg = GemmCfg<BN>;
-  const int grid = gemm_grid(M, N, K, BN, num_sms);
-  return launch_pdl(gemm_tc_kernel<BN>, dim3(grid), dim3(192), Cfg::SMEM_BYTES, st, tmA, tmB, tmC, M, N, K, ep, ws,
+  GemmEpilogue e = ep;
+  const int grid = gemm_grid(M, N, K, BN, num_sms, e);
+  return launch_pdl(gemm_tc_kernel<BN>, dim3(grid), dim3(192), Cfg::SMEM_BYTES, st, tmA, tmB, tmC, M, N, K, e, ws,
                     err);
 }
 
 // Pairs for the 2-CTA kernel: the 1-CTA rule applied to 256 x 256 pair-tiles
 // and half the SMs.
-static int gemm2_pairs(int M, int N, int K, int num_sms) { return gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2); }
+static int gemm2_pairs(int M, int N, int K, int num_sms, GemmEpilogue& ep) {
+  return gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2, ep);
+}
 
 cudaError_t gemm_prepare() {
   cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1011,9 +1084,10 @@ cudaError_t gemm_prepare() {
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,
                         const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st) {
   if (M > 128 && N % 256 == 0 && g_gemm_pairs_enabled) {
-    const int pairs = gemm2_pairs(M, N, K, num_sms);
+    GemmEpilogue e = ep;
+    const int pairs = gemm2_pairs(M, N, K, num_sms, e);
     return launch_pdl(gemm_tc2_kernel, dim3(2 * pairs), dim3(192), Gemm2Cfg::SMEM_BYTES, st, tmA, tmB, tmC, M, N, K,
-                      ep, ws, err);
+                      e, ws, err);
   }
   if (gemm_block_n(N, ep.mode) == 256)
     return launch_gemm_bn<256>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);

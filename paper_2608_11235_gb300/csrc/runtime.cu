@@ -397,7 +397,7 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr) {
     launch_rmsnorm(s->h, m->attn_norm[l], s->xn, M, d, c.norm_eps, st);
     REC(CORA_KIND_RMSNORM);
     GemmEpilogue e1{s->qkv, m->n_qkv, CORA_EPI_ROPE_BF16, s->rope, s->S, c.head_dim,
-                    (c.n_heads + c.n_kv_heads) * c.head_dim};
+                    (c.n_heads + c.n_kv_heads) * c.head_dim, 1};
     CK(launch_gemm(s->tm_xn, m->tm_qkv[l], s->tmo_qkv, M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_QKV);
     if (c.head_dim == 128) {
@@ -406,13 +406,13 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr) {
       launch_attention(s->qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, st);
     }
     REC(CORA_KIND_ATTENTION);
-    GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0};
+    GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0, 1};
     CK(launch_gemm(s->tm_attn, m->tm_o[l], s->tmo_h, M, d, c.n_heads * c.head_dim, e2, s->gemm_ws, err, m->num_sms,
                    st));
     REC(CORA_KIND_GEMM_O);
     launch_rmsnorm(s->h, m->ffn_norm[l], s->xn, M, d, c.norm_eps, st);
     REC(CORA_KIND_RMSNORM);
-    GemmEpilogue e3{s->act, m->f_pad, CORA_EPI_SWIGLU, nullptr, 0, 0, 0};
+    GemmEpilogue e3{s->act, m->f_pad, CORA_EPI_SWIGLU, nullptr, 0, 0, 0, 1};
     CK(launch_gemm(s->tm_xn, m->tm_gu[l], s->tmo_act, M, 2 * m->f_pad, d, e3, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_GATE_UP);
     CK(launch_gemm(s->tm_act, m->tm_down[l], s->tmo_h, M, d, m->f_pad, e2, s->gemm_ws, err, m->num_sms, st));
@@ -772,7 +772,7 @@ extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32
   if (!make_tmap_bf16_2d(&ta, A, M, K, size_t(K) * 2, 128, 64) || !make_tmap_bf16_2d(&tb, B, N, K, size_t(K) * 2, 128, 64) ||
       !make_gemm_out_tmap(&tc, C, M, ldc, epilogue))
     return fail(CORA_ECUDA, "cora_op_gemm: tensor map encoding failed");
-  GemmEpilogue ep{C, ldc, epilogue, rope, seq, head_dim, rope_cols};
+  GemmEpilogue ep{C, ldc, epilogue, rope, seq, head_dim, rope_cols, 0};
   CK(launch_gemm(ta, tb, tc, M, N, K, ep, dc->gemm_ws, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
   return CORA_OK;
 }

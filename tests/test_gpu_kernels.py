@@ -86,7 +86,8 @@ def run_gemm(A, Bm, M, N, K, epi, out_cols, out_dtype=torch.int16, C0=None, **kw
 
 
 @pytest.mark.parametrize("M,N,K", [(300, 512, 320), (128, 384, 64), (2048, 4096, 256), (256, 256, 4096),
-                                   (96, 768, 256), (1, 256, 128), (512, 4096, 4096), (512, 12288, 1024)])
+                                   (96, 768, 256), (1, 256, 128), (512, 4096, 4096), (512, 12288, 1024),
+                                   (96, 768, 2048)])
 def test_gemm_store(M, N, K):
     A = bits(2, 10, (M, K), 1.0)
     Bm = bits(2, 11, (N, K), 1.0 / math.sqrt(K))
@@ -94,8 +95,9 @@ def test_gemm_store(M, N, K):
     close_bf16(from_dev_bf16(Ct), f64(A) @ f64(Bm).T)
 
 
-def test_gemm_stream_k_is_deterministic():
-    M, N, K = 512, 4096, 4096          # 64 tiles of 64 k-blocks: every tile split across ~3 CTAs
+@pytest.mark.parametrize("M,N,K", [(512, 4096, 4096),    # 32 pair-tiles: two skewed k-splits each
+                                   (512, 12288, 4096)])  # 96 pair-tiles over the SM pairs: stream-K
+def test_gemm_split_tiles_are_deterministic(M, N, K):
     A = bits(2, 20, (M, K), 1.0)
     Bm = bits(2, 21, (N, K), 1.0 / math.sqrt(K))
     c1 = run_gemm(A, Bm, M, N, K, cora.EPI_STORE_BF16, N).cpu().numpy()

@@ -1,8 +1,8 @@
 """The allocation-free Eq. 1 reduction matches the regular one.
 
 cora_reduce_top1_noalloc exists for callers that cannot allocate device
-memory when they call it (for example during CUDA graph capture, or when
-their memory pool already owns the device): its scratch is a fixed array
+memory when they call it (their memory pool already owns the device, or
+their loop must not enter the allocator): its scratch is a fixed array
 inside the library.  This test calls it through the C ABI twice in a row
 (the second call reuses the array the first one left behind) and compares
 each result with cora_reduce_top1 on the same logits, within the tolerance
