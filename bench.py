@@ -44,7 +44,11 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM bytes (read + write) per launch from one ncu capture of each kernel on
 # the LLaDA-8B-shaped workload (2-layer model, same per-launch shapes), keyed
 # by a hash of the kernel source at capture time; null once the source changed.
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {
+    # gemm_tc2_kernel, mean of the QKV / O / gate-up / down launches (read + write):
+    # (125.8 + 46.3 + 244.0 + 126.1) MB / 4, profiles/gemm_tc2_llada8b_256.md
+    ("gemm", "7755988f36ea"): 135_563_000,
+}
 
 
 def load_peaks():
@@ -313,7 +317,7 @@ def run_cora(args, cfg, ws, rank, local):
     kernels = {k: {"launches_per_pass": len(v), "ms_per_launch": round(sum(v) / len(v), 5),
                    "share": round(sum(v) / step_ms, 4)} for k, v in sorted(by.items())}
     traffic = NCU_TRAFFIC.get(("gemm", src_hash("gemm.cu")))
-    roofline = {"bound": "tensor", "kernel": "gemm_tc_kernel (QKV+RoPE, O+res, gate/up+SwiGLU, down+res)",
+    roofline = {"bound": "tensor", "kernel": "gemm_tc2_kernel (QKV+RoPE, O+res, gate/up+SwiGLU, down+res)",
                 "achieved": round(gemm_tflops, 2), "peak": peak_tf, "unit": "TFLOP/s",
                 "frac": round(gemm_tflops / peak_tf, 4), "traffic": traffic,
                 "peak_source": f"{peak_src} bf16 sustained", "flops_per_launch": round(gemm_flops / n_gemm),
@@ -323,8 +327,10 @@ def run_cora(args, cfg, ws, rank, local):
                          "peak": peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]),
                          "frac": round(head_gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]), 4),
                          "bytes_per_launch": costs["lm_head_top1_bytes"], "ms_per_launch": round(head_ms, 5)},
-        "attention": {"bound": "tensor(mma.sync)", "achieved": round(costs["attention"] / (attn_ms * 1e-3) / 1e12, 2),
-                      "unit": "TFLOP/s", "ms_per_launch": round(attn_ms, 5)},
+        "attention": {"bound": "tensor", "kernel": "attention_tc_kernel" if cfg["head_dim"] == 128 else "attention_kernel",
+                      "achieved": round(costs["attention"] / (attn_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s",
+                      "peak": peak_tf, "frac": round(costs["attention"] / (attn_ms * 1e-3) / 1e12 / peak_tf, 4),
+                      "ms_per_launch": round(attn_ms, 5)},
         "pass_model_tflops": round((gemm_flops + costs["attention"] * len(by["attention"]) +
                                     costs["lm_head_top1_flops"]) / (step_ms * 1e-3) / 1e12, 2),
     }
