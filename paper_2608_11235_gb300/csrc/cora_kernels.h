@@ -109,6 +109,7 @@ struct GemmEpilogue {
   // skew toward the finishing piece, in k-blocks.
   int splits;
   int split_skew;
+  int split_pair;  // 1: two k-pieces per tile, each finalising half of the columns
 };
 
 // Stream-K workspace: one fp32 partial slot of 128 x 256 per CTA plus one

@@ -257,7 +257,6 @@ __device__ __forceinline__ void bulk_wait_read() {
   asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
 }
 
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 // Next staging buffer, once the TMA operation that last read it is done.
 __device__ __forceinline__ uint8_t* stage_acquire(Stager& sg) {
@@ -302,14 +301,16 @@ __device__ __forceinline__ void stage_issue(const Stager& sg, const CUtensorMap*
 }
 
 // Epilogue of one 128 x BN tile for this warp's 32 rows (row0 = first global
-// row of the warp's box).
+// row of the warp's box).  STORE and RESID write tile columns [c_lo, c_hi)
+// only (multiples of 64); the other modes always write the whole tile.
 template <int BN>
 __device__ __forceinline__ void gemm_epilogue_warp(const GemmEpilogue& ep, const CUtensorMap* tmC, uint32_t tacc,
-                                                   int row0, int n0, const Partials& pp, Stager& sg) {
+                                                   int row0, int n0, const Partials& pp, Stager& sg, int c_lo = 0,
+                                                   int c_hi = BN) {
   const int lane = sg.lane;
   if (ep.mode == CORA_EPI_STORE_BF16) {
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 64) {
+    for (int c = c_lo; c < c_hi; c += 64) {
       float v[4][16];
       const int cols[4] = {c, c + 16, c + 32, c + 48};
       load_acc64(tacc, cols, pp, v);
@@ -320,7 +321,7 @@ __device__ __forceinline__ void gemm_epilogue_warp(const GemmEpilogue& ep, const
     }
   } else if (ep.mode == CORA_EPI_RESID_F32) {
 #pragma unroll 1
-    for (int c = 0; c < BN; c += 64) {
+    for (int c = c_lo; c < c_hi; c += 64) {
       float v[4][16];
       const int cols[4] = {c, c + 16, c + 32, c + 48};
       load_acc64(tacc, cols, pp, v);
@@ -434,6 +435,46 @@ __device__ __forceinline__ bool wait_flag(const int* flag, volatile int* abort, 
     }
     __nanosleep(100);
   }
+  return true;
+}
+
+// Paired fix-up of a tile split into two k-pieces: each piece finalises half
+// of the tile's columns.  This writes the accumulator columns
+// [give_lo, give_lo + BN/2) that the other piece finalises into this piece's
+// slot, raises this piece's flag and waits for the other's, so the caller can
+// add the other piece's slot over its own half.  Both pieces are resident
+// (one CTA per SM, grid <= SMs) and the wait is bounded.  With two terms the
+// sum is the same whichever piece adds it, so results stay deterministic.
+template <int BN>
+__device__ __forceinline__ bool pair_exchange(uint32_t tacc, int give_lo, float* my_slot, int* my_flag,
+                                              const int* other_flag, int row_local, int etid,
+                                              volatile int* abort_flag, int* err) {
+  Partials none;
+  none.n = 0;
+  none.row = row_local;
+  none.in_smem = false;
+#pragma unroll 1
+  for (int c = give_lo; c < give_lo + BN / 2; c += 64) {
+    float v[4][16];
+    const int cols[4] = {c, c + 16, c + 32, c + 48};
+    load_acc64(tacc, cols, none, v);
+    float4* dst = reinterpret_cast<float4*>(my_slot);
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        dst[part_f4(c + 16 * q, i, row_local)] =
+            make_float4(v[q][4 * i], v[q][4 * i + 1], v[q][4 * i + 2], v[q][4 * i + 3]);
+  }
+  __threadfence();
+  named_bar_sync(1, 128);
+  bool fok = true;
+  if (etid == 0) {
+    atomicExch(my_flag, 1);
+    fok = wait_flag(other_flag, abort_flag, err);
+  }
+  if (named_bar_or(1, 128, !fok)) return false;
+  (void)ld_acquire(other_flag);
   return true;
 }
 
@@ -579,6 +620,25 @@ __global__ void __launch_bounds__(192, 1)
       tc_fence_after();
       const int mb = t / num_n, nb = t - mb * num_n;
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * BN;
+      if (ep.split_pair) {
+        // Two k-pieces per tile (CTA 2t + s): piece s finalises columns
+        // [s BN/2, (s+1) BN/2).
+        const int me = blockIdx.x, other = blockIdx.x ^ 1, s = blockIdx.x & 1;
+        if (!pair_exchange<BN>(tacc, (1 - s) * (BN / 2), ws.partial + static_cast<int64_t>(me) * kBM * BN,
+                               ws.flags + me, ws.flags + other, row_local, etid, abort_flag, err))
+          break;
+        Partials pp;
+        pp.n = 1;
+        pp.row = row_local;
+        pp.in_smem = false;
+        pp.slots[0] = ws.partial + static_cast<int64_t>(other) * kBM * BN;
+        gemm_epilogue_warp<BN>(ep, &tmC, tacc, mb * kBM + sub * 32, nb * BN, pp, sg, s * (BN / 2), (s + 1) * (BN / 2));
+        tc_fence_before();
+        mbar_arrive(&tempty[acc]);
+        named_bar_sync(1, 128);  // every thread has read the other piece's slot
+        if (etid == 0) atomicExch(ws.flags + other, 0);
+        continue;
+      }
       if (kb0 > 0) {
         // Contributor: hand the partial accumulator to the tile's finisher.
         float* slot = ws.partial + static_cast<int64_t>(blockIdx.x) * kBM * BN;
@@ -659,7 +719,10 @@ __global__ void __launch_bounds__(192, 1)
           for (int c = c_first; c <= c_last; ++c) atomicExch(ws.flags + c, 0);
       }
     }
-    if (lane == 0) bulk_wait_all();  // staged outputs fully written before the CTA retires
+    // The staging buffers must be read out before the CTA retires; the
+    // global writes themselves complete with the grid (and are visible to a
+    // dependent grid after its griddepcontrol.wait).
+    if (lane == 0) bulk_wait_read<0>();
     __syncwarp();
   }
 
@@ -907,6 +970,28 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
       tc_fence_after();
       const int mb = t / num_n, nb = t - mb * num_n;
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * BN;
+      const int row0 = mb * 256 + static_cast<int>(rank) * 128 + sub * 32;
+      if (ep.split_pair) {
+        // Two k-pieces per pair-tile (pair 2t + s): piece s finalises columns
+        // [s BN/2, (s+1) BN/2); CTA r of a pair exchanges with CTA r of the other.
+        const int s = pair & 1;
+        const int other = 2 * (pair ^ 1) + static_cast<int>(rank);
+        if (!pair_exchange<BN>(tacc, (1 - s) * (BN / 2), ws.partial + static_cast<int64_t>(me) * kBM * BN,
+                               ws.flags + me, ws.flags + other, row_local, etid, abort_flag, err))
+          break;
+        Partials pp;
+        pp.n = 1;
+        pp.row = row_local;
+        pp.in_smem = false;
+        pp.slots[0] = ws.partial + static_cast<int64_t>(other) * kBM * BN;
+        gemm_epilogue_warp<BN>(ep, &tmC, tacc, row0, nb * BN, pp, sg, s * (BN / 2), (s + 1) * (BN / 2));
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive_remote(lead_tempty[acc]);
+        named_bar_sync(1, 128);  // every thread has read the other piece's slot
+        if (etid == 0) atomicExch(ws.flags + other, 0);
+        continue;
+      }
       if (kb0 > 0) {
         // Contributor: hand this CTA's 128-row partial to the tile's finisher.
         float* slot = ws.partial + static_cast<int64_t>(me) * kBM * BN;
@@ -978,7 +1063,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
         }
         if (n_c > 4) record_error(err, CORA_DERR_SPLIT_WAIT);
       }
-      gemm_epilogue_warp<BN>(ep, &tmC, tacc, mb * 256 + static_cast<int>(rank) * 128 + sub * 32, nb * BN, pp, sg);
+      gemm_epilogue_warp<BN>(ep, &tmC, tacc, row0, nb * BN, pp, sg);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(lead_tempty[acc]);
@@ -988,7 +1073,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
           for (int c = c_first; c <= c_last; ++c) atomicExch(ws.flags + 2 * c + static_cast<int>(rank), 0);
       }
     }
-    if (lane == 0) bulk_wait_all();
+    if (lane == 0) bulk_wait_read<0>();  // staging read out (see the 1-CTA kernel)
     __syncwarp();
   }
 
@@ -1032,6 +1117,7 @@ static int gemm_grid(int M, int N, int K, int bn, int num_sms, GemmEpilogue& ep)
   const long long W = static_cast<long long>(tiles) * KB;
   ep.splits = 0;
   ep.split_skew = 0;
+  ep.split_pair = 0;
   if (2 * tiles <= num_sms) {
     // Few tiles: split every tile into the same number of k-ranges (at most
     // 4), so each CTA holds one piece and every finisher has its operand
@@ -1039,7 +1125,11 @@ static int gemm_grid(int M, int N, int K, int bn, int num_sms, GemmEpilogue& ep)
     int splits = num_sms / tiles;
     if (splits > 4) splits = 4;
     if (splits > KB) splits = KB;
-    if (splits >= 2 && KB % splits == 0) {
+    if (splits == 2 && (ep.mode == CORA_EPI_STORE_BF16 || ep.mode == CORA_EPI_RESID_F32)) {
+      // Both pieces share the fix-up, each finalising half of the columns.
+      ep.splits = 2;
+      ep.split_pair = 1;
+    } else if (splits >= 2 && KB % splits == 0) {
       int skew = (kSkewTotal + splits - 1) / splits;
       if (skew > KB / (2 * splits)) skew = KB / (2 * splits);
       ep.splits = splits;

@@ -87,7 +87,7 @@ def run_gemm(A, Bm, M, N, K, epi, out_cols, out_dtype=torch.int16, C0=None, **kw
 
 @pytest.mark.parametrize("M,N,K", [(300, 512, 320), (128, 384, 64), (2048, 4096, 256), (256, 256, 4096),
                                    (96, 768, 256), (1, 256, 128), (512, 4096, 4096), (512, 12288, 1024),
-                                   (96, 768, 2048)])
+                                   (96, 768, 2048), (128, 16384, 512)])
 def test_gemm_store(M, N, K):
     A = bits(2, 10, (M, K), 1.0)
     Bm = bits(2, 11, (N, K), 1.0 / math.sqrt(K))
@@ -105,7 +105,7 @@ def test_gemm_split_tiles_are_deterministic(M, N, K):
     assert np.array_equal(c1, c2)
 
 
-@pytest.mark.parametrize("M,N,K", [(300, 512, 320), (130, 256, 1024), (512, 4096, 12288)])
+@pytest.mark.parametrize("M,N,K", [(300, 512, 320), (130, 256, 1024), (512, 4096, 12288), (100, 16384, 512)])
 def test_gemm_residual(M, N, K):
     A = bits(3, 10, (M, K), 1.0)
     Bm = bits(3, 11, (N, K), 1.0 / math.sqrt(K))
