@@ -4,16 +4,23 @@
 //
 // Per key tile j:
 //   S_j = Q K_j^T        tcgen05.mma M=128 (queries) x N=128 (keys) x K=128 (hd), TMEM
-//   softmax              warps 2..5, one query row per thread: running max m and
-//                        sum l (base 2, scores pre-scaled by log2(e)/sqrt(hd)),
-//                        P_j = exp2(S_j - m_j) written to shared memory as bf16
-//   O_j' = P_j V_j       tcgen05.mma M=128 x N=128 (hd) x K=128 (keys), V read as an
-//                        MN-major operand straight from its [keys][hd] layout
-//   O = a_j O + O_j'     in registers (a_j = exp2(m_{j-1} - m_j)), one row per thread
-// Two TMEM buffers each for S and O' (512 columns) and two P buffers let the
-// softmax of tile j overlap the MMAs of tiles j-1 and j+1.
-// Warps: 0 = TMA producer, 1 = TMEM allocator + MMA issuer, 2..5 = softmax.
-// Keys beyond the sequence end are masked; queries beyond it are not stored.
+//   softmax              warps 2..5, one query row per thread: the row of S_j is
+//                        read from TMEM once; P_j = exp2(S_j - m) (base 2,
+//                        scores pre-scaled by log2(e)/sqrt(hd)) goes to shared
+//                        memory as bf16 and the row sum l accumulates
+//   O += P_j V_j         tcgen05.mma M=128 x N=128 (hd) x K=128 (keys) into one
+//                        TMEM accumulator; V is read as an MN-major operand
+//                        straight from its [keys][hd] layout
+// The reference max m of a row is raised only when a tile's max exceeds it by
+// more than 2^8 (then O and l are rescaled in place, after the previous PV
+// has completed).  The final O / l is the same for any choice of m, and
+// P <= 2^8 keeps full bf16 precision, so the result is unchanged while the
+// softmax warps never wait for a PV in the common case.
+// Two TMEM buffers for S and two P buffers let the softmax of tile j overlap
+// the MMAs of tiles j-1 and j+1.  TMEM: S[0] +0, S[1] +128, O +256.
+// Warps: 0 = TMA producer, 1 = TMEM allocator + MMA issuer, 2..5 = softmax and
+// output.  Keys beyond the sequence end are masked; the output is written by
+// TMA through a [sequence][row][column] map, which clips rows beyond the end.
 #include <math.h>
 
 #include "cora_device.cuh"
@@ -27,6 +34,7 @@ constexpr int KT = 128;          // keys per tile
 constexpr int HD = 128;          // head dim
 constexpr int OPND = QT * HD * 2;  // 32 KB: one 128 x 128 bf16 operand (two 16 KB swizzle columns)
 constexpr int SMEM = 7 * OPND + 1024 + 256;  // Q, K[2], V[2], P[2]
+constexpr float kRescale = 8.0f; // log2 headroom before the reference max is raised
 }  // namespace attn
 
 // MN-major (N contiguous) 128-byte-swizzled operand: 8-row K groups 1024 B
@@ -41,15 +49,39 @@ __device__ __forceinline__ uint64_t sw128_mnmajor_desc(uint32_t smem_addr, uint3
   return d;
 }
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
-  float a[16], b[16];
-  tmem_ld16x2(taddr, taddr + 16, a, b);
-#pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    v[i] = a[i];
-    v[16 + i] = b[i];
-  }
+// Load 128 consecutive fp32 columns of this warp's 32 TMEM lanes (one lane
+// per thread) and wait for them, in one statement so that no register is
+// read before the load has landed.
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, uint32_t (&r)[128]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x128.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63,%64,%65,%66,%67,%68,%69,%70,%71,%72,%73,%74,%75,%76,%77,%78,%79,%80,%81,%82,%83,%84,%85,%86,%87,%88,%89,%90,%91,%92,%93,%94,%95,%96,%97,%98,%99,%100,%101,%102,%103,%104,%105,%106,%107,%108,%109,%110,%111,%112,%113,%114,%115,%116,%117,%118,%119,%120,%121,%122,%123,%124,%125,%126,%127}, [%128];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63]), "=r"(r[64]), "=r"(r[65]), "=r"(r[66]), "=r"(r[67]), "=r"(r[68]), "=r"(r[69]), "=r"(r[70]), "=r"(r[71]), "=r"(r[72]), "=r"(r[73]), "=r"(r[74]), "=r"(r[75]), "=r"(r[76]), "=r"(r[77]), "=r"(r[78]), "=r"(r[79]), "=r"(r[80]), "=r"(r[81]), "=r"(r[82]), "=r"(r[83]), "=r"(r[84]), "=r"(r[85]), "=r"(r[86]), "=r"(r[87]), "=r"(r[88]), "=r"(r[89]), "=r"(r[90]), "=r"(r[91]), "=r"(r[92]), "=r"(r[93]), "=r"(r[94]), "=r"(r[95]), "=r"(r[96]), "=r"(r[97]), "=r"(r[98]), "=r"(r[99]), "=r"(r[100]), "=r"(r[101]), "=r"(r[102]), "=r"(r[103]), "=r"(r[104]), "=r"(r[105]), "=r"(r[106]), "=r"(r[107]), "=r"(r[108]), "=r"(r[109]), "=r"(r[110]), "=r"(r[111]), "=r"(r[112]), "=r"(r[113]), "=r"(r[114]), "=r"(r[115]), "=r"(r[116]), "=r"(r[117]), "=r"(r[118]), "=r"(r[119]), "=r"(r[120]), "=r"(r[121]), "=r"(r[122]), "=r"(r[123]), "=r"(r[124]), "=r"(r[125]), "=r"(r[126]), "=r"(r[127])
+      : "r"(taddr)
+      : "memory");
 }
+
+// Load 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one lane
+// per thread) and wait for them, in one statement so that no register is
+// read before the load has landed.
+__device__ __forceinline__ void tmem_ld32w(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+}
+
+// Store 32 consecutive fp32 columns of this warp's 32 TMEM lanes.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};"
+               :
+               : "r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 __device__ __forceinline__ float ex2f(float x) {
   float y;
@@ -57,9 +89,16 @@ __device__ __forceinline__ float ex2f(float x) {
   return y;
 }
 
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0, int c1, int c2) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
+               : "memory");
+}
+
 __global__ void __launch_bounds__(192, 1)
-    attention_tc_kernel(const __grid_constant__ CUtensorMap tmQKV, uint16_t* __restrict__ out, int S, int Hq, int Hkv,
-                        int* err) {
+    attention_tc_kernel(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ CUtensorMap tmOut, int S,
+                        int Hq, int Hkv, int* err) {
   using namespace attn;
   // idesc: M = 128, N = 128, bf16 x bf16 -> f32; PV reads B (V) MN-major.
   constexpr uint32_t IDESC_QK = idesc_bf16_f32(128, 128);
@@ -73,15 +112,13 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t* sP[2] = {smem + 5 * OPND, smem + 6 * OPND};
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 7 * OPND);
   uint64_t* qfull = bars + 0;
-  uint64_t* kvfull = bars + 1;   // [2]
-  uint64_t* kvempty = bars + 3;  // [2]
-  uint64_t* sfull = bars + 5;    // [2]
-  uint64_t* sfree = bars + 7;    // [2]
-  uint64_t* pfull = bars + 9;    // [2]
-  uint64_t* pfree = bars + 11;   // [2]
-  uint64_t* ofull = bars + 13;   // [2]
-  uint64_t* ofree = bars + 15;   // [2]
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
+  uint64_t* kvfull = bars + 1;   // [2] K_j, V_j landed
+  uint64_t* kvempty = bars + 3;  // [2] QK_j and PV_j done with K_j, V_j
+  uint64_t* sfull = bars + 5;    // [2] S_j in TMEM
+  uint64_t* sfree = bars + 7;    // [2] S_j read out by the four softmax warps
+  uint64_t* pfull = bars + 9;    // [2] P_j written (and O rescaled, if it was)
+  uint64_t* pdone = bars + 11;   // [2] PV_j complete (P buffer free, O up to date)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 13);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -100,22 +137,24 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(&sfull[i], 1);
       mbar_init(&sfree[i], 4);
       mbar_init(&pfull[i], 4);
-      mbar_init(&pfree[i], 1);
-      mbar_init(&ofull[i], 1);
-      mbar_init(&ofree[i], 4);
+      mbar_init(&pdone[i], 1);
     }
     *abort_flag = 0;
     fence_barrier_init();
   }
-  if (warp == 0 && lane == 0) tma_prefetch_desc(&tmQKV);
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmQKV);
+    tma_prefetch_desc(&tmOut);
+  }
   if (warp == 1) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
+  __syncwarp();  // converged arrival (one lane of warp 0 initialised the barriers)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem_base = *tmem_slot;  // S[0] at +0, S[1] at +128, O'[0] at +256, O'[1] at +384
+  const uint32_t tmem_base = *tmem_slot;
   pdl_trigger();
   pdl_wait();
 
@@ -139,25 +178,22 @@ __global__ void __launch_bounds__(192, 1)
     if (lane == 0) {
       bool ok = mbar_wait(qfull, 0, abort_flag, err, CORA_DERR_MMA_WAIT);
       const uint32_t q_addr = smem_u32(sQ);
-      // PV of tile jj: O'[jj%2] = P[jj%2] V[jj%2].
+      const uint32_t o_tmem = tmem_base + 256;
+      // O += P_jj V_jj.
       auto issue_pv = [&](int jj) -> bool {
         const int s = jj & 1;
-        const uint32_t ph = (jj >> 1) & 1;
-        if (!mbar_wait(&pfull[s], ph, abort_flag, err, CORA_DERR_MMA_WAIT)) return false;
-        if (!mbar_wait(&ofree[s], ph ^ 1u, abort_flag, err, CORA_DERR_MMA_WAIT)) return false;
+        if (!mbar_wait(&pfull[s], (jj >> 1) & 1, abort_flag, err, CORA_DERR_MMA_WAIT)) return false;
         tc_fence_after();
         const uint32_t p_addr = smem_u32(sP[s]), v_addr = smem_u32(sV[s]);
-        const uint32_t d = tmem_base + 256 + s * 128;
 #pragma unroll
         for (int k = 0; k < KT / 16; ++k) {
           // A = P: K-major, keys contiguous, 64-key swizzle columns 16 KB apart.
           const uint64_t a = sw128_kmajor_desc(p_addr + (k >> 2) * (OPND / 2) + (k & 3) * 32);
           // B = V: rows are keys (K), 64-element hd blocks 16 KB apart (MN-major).
           const uint64_t bd = sw128_mnmajor_desc(v_addr + k * 16 * 128, OPND / 2);
-          umma_bf16(d, a, bd, IDESC_PV, k > 0);
+          umma_bf16(o_tmem, a, bd, IDESC_PV, (jj > 0 || k > 0) ? 1u : 0u);
         }
-        umma_commit(&ofull[s]);
-        umma_commit(&pfree[s]);
+        umma_commit(&pdone[s]);
         umma_commit(&kvempty[s]);
         return true;
       };
@@ -183,120 +219,114 @@ __global__ void __launch_bounds__(192, 1)
     const int sub = warp & 3;
     const int r = sub * 32 + lane;  // query row within the tile (TMEM lane)
     const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
+    const uint32_t o_lane = lane_base + 256;
     const float sl2 = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
-    float o[HD];
-#pragma unroll
-    for (int i = 0; i < HD; ++i) o[i] = 0.f;
-    float m = -INFINITY, l = 0.f, a_prev = 1.f;
+    float m = -INFINITY, l = 0.f;
     bool ok = true;
-    for (int j = 0; j <= n_kt && ok; ++j) {
-      if (j < n_kt) {
-        const int s = j & 1;
-        const uint32_t ph = (j >> 1) & 1;
-        ok = mbar_wait(&sfull[s], ph, abort_flag, err, CORA_DERR_EPI_WAIT);
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t sb = lane_base + s * 128;
-        const int kbase = j * KT;
-        // pass 1: row max
-        float mx = m;
-#pragma unroll 1
-        for (int c = 0; c < KT; c += 32) {
-          float v[32];
-          tmem_ld32(sb + c, v);
+    for (int j = 0; j < n_kt && ok; ++j) {
+      const int s = j & 1;
+      const uint32_t ph = (j >> 1) & 1;
+      ok = mbar_wait(&sfull[s], ph, abort_flag, err, CORA_DERR_EPI_WAIT);
+      if (!ok) break;
+      tc_fence_after();
+      uint32_t v[128];
+      tmem_ld128(lane_base + s * 128, v);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sfree[s]);  // S buffer may take S_{j+2}
+      const int kbase = j * KT;
+      float mx = -INFINITY;
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float x = (kbase + c + i < S) ? v[i] * sl2 : -INFINITY;
-            mx = fmaxf(mx, x);
-          }
-        }
-        const float alpha = ex2f(m - mx);  // 0 on the first tile (m = -inf)
-        m = mx;
-        // P buffer s is free once the PV of tile j-2 has read it.
-        if (j >= 2) ok = mbar_wait(&pfree[s], ph ^ 1u, abort_flag, err, CORA_DERR_EPI_WAIT);
-        if (!ok) break;
-        // pass 2: P = exp2(S - m) as bf16 into the K-major swizzled P tile
-        float rs = 0.f;
-        uint8_t* prow = sP[s];
-#pragma unroll 1
-        for (int c = 0; c < KT; c += 32) {
-          float v[32];
-          tmem_ld32(sb + c, v);
-          uint32_t pk[16];
-#pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const float x0 = (kbase + c + 2 * i < S) ? ex2f(fmaf(v[2 * i], sl2, -m)) : 0.f;
-            const float x1 = (kbase + c + 2 * i + 1 < S) ? ex2f(fmaf(v[2 * i + 1], sl2, -m)) : 0.f;
-            rs += x0 + x1;
-            pk[i] = pack_bf16x2(x0, x1);
-          }
-          // keys c .. c+31 -> swizzle column c/64, 16-byte chunks (c%64)/8 .. +3
-#pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const int key = c + 8 * q;
-            const int chunk = (key & 63) >> 3;
-            uint8_t* dst = prow + (key >> 6) * (OPND / 2) + r * 128 + ((chunk ^ (r & 7)) << 4);
-            *reinterpret_cast<uint4*>(dst) = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-          }
-        }
-        l = l * alpha + rs;
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&sfree[s]);
-          mbar_arrive(&pfull[s]);
-        }
-        // fold O'_{j-1} (computed with the previous max) into the row
-        if (j >= 1) {
+      for (int i = 0; i < KT; ++i) {
+        if (kbase + i >= S) v[i] = __float_as_uint(-INFINITY);
+        mx = fmaxf(mx, __uint_as_float(v[i]));
+      }
+      mx *= sl2;
+      const bool raise = mx > m + kRescale;
+      if (__any_sync(0xffffffffu, raise)) {
+        const float m_new = raise ? mx : m;
+        const float a = ex2f(m - m_new);  // 0 on the first tile, 1 where not raised
+        l *= a;
+        m = m_new;
+        if (j > 0) {
+          // O holds PV_0 .. PV_{j-1}: wait for the last one, then rescale in place.
           const int sp = (j - 1) & 1;
-          const uint32_t php = ((j - 1) >> 1) & 1;
-          ok = mbar_wait(&ofull[sp], php, abort_flag, err, CORA_DERR_EPI_WAIT);
+          ok = mbar_wait(&pdone[sp], ((j - 1) >> 1) & 1, abort_flag, err, CORA_DERR_EPI_WAIT);
           if (!ok) break;
           tc_fence_after();
-          const uint32_t ob = lane_base + 256 + sp * 128;
-#pragma unroll
+#pragma unroll 1
           for (int c = 0; c < HD; c += 32) {
-            float v[32];
-            tmem_ld32(ob + c, v);
+            uint32_t o[32];
+            tmem_ld32w(o_lane + c, o);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[c + i] = o[c + i] * a_prev + v[i];
+            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * a);
+            tmem_st32(o_lane + c, o);
           }
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&ofree[sp]);
+          tmem_wait_st();
         }
-        a_prev = alpha;  // applied to O when O'_j is folded in at the next iteration
-      } else {
-        // after the last tile: fold O'_{n-1}
-        const int sp = (j - 1) & 1;
-        const uint32_t php = ((j - 1) >> 1) & 1;
-        ok = mbar_wait(&ofull[sp], php, abort_flag, err, CORA_DERR_EPI_WAIT);
-        if (!ok) break;
-        tc_fence_after();
-        const uint32_t ob = lane_base + 256 + sp * 128;
-#pragma unroll
-        for (int c = 0; c < HD; c += 32) {
-          float v[32];
-          tmem_ld32(ob + c, v);
-#pragma unroll
-          for (int i = 0; i < 32; ++i) o[c + i] = o[c + i] * a_prev + v[i];
-        }
-        tc_fence_before();
       }
+      // P buffer s is free once PV_{j-2} has read it.
+      if (j >= 2) ok = mbar_wait(&pdone[s], ph ^ 1u, abort_flag, err, CORA_DERR_EPI_WAIT);
+      if (!ok) break;
+      float rs = 0.f;
+      uint8_t* prow = sP[s];
+#pragma unroll
+      for (int c = 0; c < KT; c += 8) {
+        uint32_t pk[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float x0 = ex2f(fmaf(__uint_as_float(v[c + 2 * i]), sl2, -m));
+          const float x1 = ex2f(fmaf(__uint_as_float(v[c + 2 * i + 1]), sl2, -m));
+          rs += x0 + x1;
+          pk[i] = pack_bf16x2(x0, x1);
+        }
+        // keys c .. c+7 -> swizzle column c/64, 16-byte chunk (c%64)/8
+        const int chunk = (c & 63) >> 3;
+        *reinterpret_cast<uint4*>(prow + (c >> 6) * (OPND / 2) + r * 128 + ((chunk ^ (r & 7)) << 4)) =
+            make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      }
+      l += rs;
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&pfull[s]);
     }
-    if (ok && q0 + r < S) {
+    // Output: wait for the last PV, O / l as bf16 into this warp's 32 rows of
+    // a free P buffer (same swizzled layout as the store map's box), then TMA.
+    if (ok) {
+      const int sl = (n_kt - 1) & 1;
+      ok = mbar_wait(&pdone[sl], ((n_kt - 1) >> 1) & 1, abort_flag, err, CORA_DERR_EPI_WAIT);
+    }
+    if (ok) {
+      tc_fence_after();
+      uint32_t o[128];
+      tmem_ld128(o_lane, o);
       const float inv = 1.f / l;
-      uint16_t* dst = out + static_cast<int64_t>(row_base + q0 + r) * (static_cast<int64_t>(Hq) * HD) + qcol;
+      uint8_t* stg = sP[0];
 #pragma unroll
       for (int c = 0; c < HD; c += 8) {
-        *reinterpret_cast<uint4*>(dst + c) =
-            make_uint4(pack_bf16x2(o[c] * inv, o[c + 1] * inv), pack_bf16x2(o[c + 2] * inv, o[c + 3] * inv),
-                       pack_bf16x2(o[c + 4] * inv, o[c + 5] * inv), pack_bf16x2(o[c + 6] * inv, o[c + 7] * inv));
+        const int chunk = (c & 63) >> 3;
+        *reinterpret_cast<uint4*>(stg + (c >> 6) * (OPND / 2) + r * 128 + ((chunk ^ (r & 7)) << 4)) = make_uint4(
+            pack_bf16x2(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
+            pack_bf16x2(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
+            pack_bf16x2(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
+            pack_bf16x2(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        for (int c = 0; c < 2; ++c)
+          tma_store_3d(&tmOut, stg + c * (OPND / 2) + sub * 32 * 128, qcol + c * 64, q0 + sub * 32, b);
+        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
       }
     }
+    tc_fence_before();
   }
 
+  // Each warp arrives converged: the producer and MMA warps ran their loops
+  // on one lane, and bar.sync counts a divergent warp's lanes separately.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -315,6 +345,13 @@ cudaError_t attention_tc_prepare() {
 
 cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int* err,
                                 cudaStream_t st) {
+  // Output map [B][S][Hq*hd] bf16, boxes of 32 rows x 64 columns (one warp's
+  // rows, one 128-byte swizzle column).
+  CUtensorMap tmOut;
+  if (!make_tmap_bf16_3d(&tmOut, out, static_cast<uint64_t>(Hq) * attn::HD, S, B,
+                         static_cast<uint64_t>(Hq) * attn::HD * 2, static_cast<uint64_t>(S) * Hq * attn::HD * 2, 64,
+                         32, 1))
+    return cudaErrorInvalidValue;
   dim3 grid((S + attn::QT - 1) / attn::QT, Hq, B);
-  return launch_pdl(attention_tc_kernel, grid, dim3(192), attn::SMEM, st, tmQKV, out, S, Hq, Hkv, err);
+  return launch_pdl(attention_tc_kernel, grid, dim3(192), attn::SMEM, st, tmQKV, tmOut, S, Hq, Hkv, err);
 }

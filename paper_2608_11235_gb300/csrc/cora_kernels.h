@@ -123,6 +123,9 @@ size_t gemm_workspace_bytes(int num_sms);
 // Tensor-map encoder (driver entry point fetched at runtime).
 bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
                        uint32_t box_rows, uint32_t box_cols);
+// 3-D bf16 map (innermost d0), 128-byte swizzle; strides of dims 1 and 2 in bytes.
+bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t stride1_bytes,
+                       uint64_t stride2_bytes, uint32_t b0, uint32_t b1, uint32_t b2);
 
 int gemm_block_n(int N, int mode);
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,

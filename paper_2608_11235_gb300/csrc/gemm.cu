@@ -529,6 +529,7 @@ __global__ void __launch_bounds__(192, 1)
     tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
     tmem_relinquish();
   }
+  __syncwarp();  // converged arrival (one lane of warp 0 initialised the barriers)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -726,6 +727,9 @@ __global__ void __launch_bounds__(192, 1)
     __syncwarp();
   }
 
+  // Each warp arrives converged: the producer and MMA warps ran their loops
+  // on one lane, and bar.sync counts a divergent warp's lanes separately.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -862,6 +866,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
   }
+  __syncwarp();  // converged arrival (one lane of warp 0 initialised the barriers)
   tc_fence_before();
   __syncthreads();
   cluster_sync_all();  // both CTAs' barriers initialised before any cross-CTA signal
@@ -1077,6 +1082,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
     __syncwarp();
   }
 
+  // Each warp arrives converged: the producer and MMA warps ran their loops
+  // on one lane, and bar.sync counts a divergent warp's lanes separately.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   cluster_sync_all();  // no cross-CTA signal is still in flight

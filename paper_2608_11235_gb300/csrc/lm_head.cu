@@ -76,6 +76,7 @@ __global__ void __launch_bounds__(192, 1)
     tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
     tmem_relinquish();
   }
+  __syncwarp();  // converged arrival (one lane of warp 0 initialised the barriers)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -196,6 +197,9 @@ __global__ void __launch_bounds__(192, 1)
     }
   }
 
+  // Each warp arrives converged: the producer and MMA warps ran their loops
+  // on one lane, and bar.sync counts a divergent warp's lanes separately.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
