@@ -266,12 +266,14 @@ def run_cora(args, cfg, ws, rank, local):
     s = cora.cora_session_create(m, B, prompt_dev, P, G, BL, T, tau, K)
     stream = torch.cuda.ExternalStream(cora.cora_session_stream(s))
 
+    device_loop = [False]
+
     def decode():
+        # one complete decode: a single graph launch whose WHILE node runs
+        # step after step until every sequence has finished
         cora.cora_session_reset(s, prompt_dev)
-        done = False
-        while not done:
-            done = cora.cora_denoise_step(s)
-        return cora.cora_session_batched_passes(s)
+        steps, device_loop[0] = cora.cora_session_run(s)
+        return steps
 
     for _ in range(args.warmup):
         passes = decode()
@@ -383,7 +385,9 @@ def run_cora(args, cfg, ws, rank, local):
                    "passes_per_seq": float(per_seq_passes.mean()),
                    "passes_per_block": round(float(per_seq_passes.mean()) / (G // BL), 3),
                    "rho": round(float(per_seq_passes.mean()) / ((G // BL) * T), 4),
-                   "parallelism": f"replicas x{ws}"},
+                   "parallelism": f"replicas x{ws}",
+                   "decode_loop": "device (one graph launch per decode, conditional WHILE node)" if device_loop[0]
+                   else "host (one graph launch per step)"},
         "e2e": {"value": round(ws * B * G * args.steps / e2e_s, 3), "unit": "tokens/s",
                 "h2d_bytes_per_step": int(B * P * 4), "d2h_bytes_per_step": int(B * G * 4 + B * 8),
                 "timing": "host wall clock around cora_generate (pinned host prompt in, host tokens out)"},

@@ -159,6 +159,18 @@ CORA_API int cora_session_reset(cora_session* s, const int32_t* prompt);
  * Errors: CORA_ESTATE (already finished), CORA_ETIMEOUT, CORA_ECUDA. */
 CORA_API int cora_denoise_step(cora_session* s, uint8_t* all_done_out);
 
+/* Runs cora_denoise_step until every sequence has finished (the decode loop
+ * of Sec. 3, Fig. 2), as ONE graph launch: a conditional WHILE node around
+ * the step, whose condition a device kernel sets after each step's gate (all
+ * sequences finished, an error, or n_blocks * T steps end it), so no host
+ * round trip separates the passes.  Where the runtime cannot build that
+ * graph, the same loop runs on the host, one cora_denoise_step at a time.
+ *   steps_out      host int32 or NULL (out): batched steps executed by this call
+ *   on_device_out  host uint8 or NULL (out): 1 when the device loop ran
+ * Synchronous.  Errors: CORA_ESTATE (already finished, or unfinished after
+ * the horizon), CORA_ETIMEOUT, CORA_ECUDA. */
+CORA_API int cora_session_run(cora_session* s, int32_t* steps_out, uint8_t* on_device_out);
+
 /* Copies session state to host buffers (any pointer may be NULL; synchronous):
  *   tokens  int32 [B, prompt_len + gen_len]   canvas
  *   state   uint8 [B, gen_len]               CORA_UNRESOLVED/TRANSFERRED/ACCEPTED
@@ -208,8 +220,8 @@ CORA_API int cora_session_stream(cora_session* s, void** out);
 CORA_API int cora_session_batched_passes(cora_session* s, int64_t* out);
 
 /* Full decode (Sec. 3, Fig. 2): creates or reuses the model's cached session
- * for these shapes, runs cora_denoise_step until every sequence has finished,
- * and copies the result to host memory.
+ * for these shapes, runs the decode with cora_session_run, and copies the
+ * result to host memory.
  *   prompt      "any" int32 [B, P]
  *   tokens_out  host int32 [B, gen_len]   generated ids
  *   passes_out  host int64 [B]            executed dense passes per sequence

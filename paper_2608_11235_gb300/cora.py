@@ -22,7 +22,7 @@ EPI_STORE_BF16, EPI_RESID_F32, EPI_SWIGLU, EPI_ROPE_BF16 = 0, 1, 2, 3
 
 EXPORTED = [
     "cora_last_error", "cora_version", "cora_model_create", "cora_model_destroy", "cora_session_create",
-    "cora_session_destroy", "cora_session_reset", "cora_denoise_step", "cora_session_read", "cora_session_write",
+    "cora_session_destroy", "cora_session_reset", "cora_denoise_step", "cora_session_run", "cora_session_read", "cora_session_write",
     "cora_session_batched_passes", "cora_generate", "cora_gate_transfer", "cora_reduce_top1", "cora_reduce_gate",
     "cora_op_gemm", "cora_op_attention", "cora_op_rmsnorm", "cora_op_lm_head_top1", "cora_synth_normal_bf16",
     "cora_device_error", "cora_session_profile_step", "cora_session_stream", "cora_reduce_top1_noalloc",
@@ -77,6 +77,7 @@ def lib():
             "cora_session_destroy": ([vp], C.c_int),
             "cora_session_reset": ([vp, vp], C.c_int),
             "cora_denoise_step": ([vp, vp], C.c_int),
+            "cora_session_run": ([vp, vp, vp], C.c_int),
             "cora_session_read": ([vp] + [vp] * 9, C.c_int),
             "cora_session_write": ([vp] + [vp] * 5, C.c_int),
             "cora_session_batched_passes": ([vp, vp], C.c_int),
@@ -177,6 +178,14 @@ def cora_denoise_step(session) -> bool:
     done = np.zeros(1, np.uint8)
     _check("cora_denoise_step", lib().cora_denoise_step(session, ptr(done)))
     return bool(done[0])
+
+
+def cora_session_run(session) -> tuple:
+    """Whole decode (one graph launch where available): (steps, on_device)."""
+    steps = np.zeros(1, np.int32)
+    dev = np.zeros(1, np.uint8)
+    _check("cora_session_run", lib().cora_session_run(session, ptr(steps), ptr(dev)))
+    return int(steps[0]), bool(dev[0])
 
 
 def cora_session_read(session, B, S, G, BL) -> dict:

@@ -121,6 +121,9 @@ struct GemmWorkspace {
 size_t gemm_workspace_bytes(int num_sms);
 
 // Tensor-map encoder (driver entry point fetched at runtime).
+// One-thread kernel that sets the WHILE condition of the whole-decode graph.
+cudaError_t launch_step_loop_cond(cudaGraphConditionalHandle h, int32_t* status, int32_t max_iters, cudaStream_t st);
+
 bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint64_t row_stride_bytes,
                        uint32_t box_rows, uint32_t box_cols);
 // 3-D bf16 map (innermost d0), 128-byte swizzle; strides of dims 1 and 2 in bytes.

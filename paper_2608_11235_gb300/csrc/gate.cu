@@ -331,6 +331,17 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
   }
 }
 
+// Loop control of the whole-decode graph (a conditional WHILE node around
+// one step): counts the pass in status[2] and keeps looping while some
+// sequence is unfinished, no kernel has recorded an error and the horizon
+// (n_blocks * T passes) is not reached.
+__global__ void step_loop_cond_kernel(cudaGraphConditionalHandle h, int32_t* status, int32_t max_iters) {
+  const int32_t it = status[2] + 1;
+  status[2] = it;
+  const bool done = reinterpret_cast<const uint8_t*>(status)[0] != 0;
+  cudaGraphSetConditional(h, (!done && status[1] == 0 && it < max_iters) ? 1u : 0u);
+}
+
 }  // namespace cora
 
 using namespace cora;
@@ -436,4 +447,9 @@ extern "C" int cora_reduce_top1_noalloc(const uint16_t* logits, int32_t rows, in
   if (cudaGetLastError() != cudaSuccess)
     return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: kernel launch failed");
   return CORA_OK;
+}
+
+cudaError_t launch_step_loop_cond(cudaGraphConditionalHandle h, int32_t* status, int32_t max_iters, cudaStream_t st) {
+  step_loop_cond_kernel<<<1, 1, 0, st>>>(h, status, max_iters);
+  return cudaGetLastError();
 }

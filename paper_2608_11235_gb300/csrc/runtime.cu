@@ -357,7 +357,9 @@ struct cora_session {
   CUtensorMap tmo_qkv{}, tmo_h{}, tmo_act{};  // GEMM output maps
   CUtensorMap tm_qkv_in{};                     // QKV as the attention kernel's TMA source
   GemmWorkspace gemm_ws{nullptr, nullptr};
-  cudaGraphExec_t graph = nullptr;
+  cudaGraphExec_t graph = nullptr;      // one step
+  cudaGraphExec_t run_graph = nullptr;  // WHILE node around one step: a whole decode (null: not available)
+  int32_t max_iters = 0;                // n_blocks * T
   int64_t batched_passes = 0;
   bool finished = false;
 };
@@ -393,7 +395,11 @@ struct LaunchRecorder {
 #define REC(kind) \
   if (rec) rec->mark(kind)
 
-static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr) {
+// One dense pass + Eq. 1 + gate.  With `loop`, the step is the body of the
+// whole-decode WHILE node: the status read-back is replaced by the kernel
+// that sets the loop condition.
+static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
+                        const cudaGraphConditionalHandle* loop = nullptr) {
   cora_model* m = s->m;
   const cora_model_config& c = m->cfg;
   const int d = c.d_model, M = s->M;
@@ -442,8 +448,46 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr) {
   launch_session_gate(ga, st);
   REC(CORA_KIND_GATE);
   CK(cudaGetLastError());
-  CK(cudaMemcpyAsync(s->status_h, s->status, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+  if (loop)
+    CK(launch_step_loop_cond(*loop, s->status, s->max_iters, st));
+  else
+    CK(cudaMemcpyAsync(s->status_h, s->status, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
   return CORA_OK;
+}
+
+// The whole decode as one graph: a conditional WHILE node whose body is one
+// step (captured into it), so no host round trip separates the passes.
+// Returns false (and leaves no graph) where the runtime does not support it.
+static bool build_run_graph(cora_session* s) {
+  cudaGraph_t g = nullptr;
+  if (cudaGraphCreate(&g, 0) != cudaSuccess) return false;
+  bool ok = false;
+  do {
+    cudaGraphConditionalHandle h;
+    if (cudaGraphConditionalHandleCreate(&h, g, 1, cudaGraphCondAssignDefault) != cudaSuccess) break;
+    cudaGraphNodeParams p{};
+    p.type = cudaGraphNodeTypeConditional;
+    p.conditional.handle = h;
+    p.conditional.type = cudaGraphCondTypeWhile;
+    p.conditional.size = 1;
+    cudaGraphNode_t node;
+    if (cudaGraphAddNode(&node, g, nullptr, nullptr, 0, &p) != cudaSuccess) break;
+    cudaGraph_t body = p.conditional.phGraph_out[0];
+    if (cudaStreamBeginCaptureToGraph(s->stream, body, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal) !=
+        cudaSuccess)
+      break;
+    const int rc = enqueue_step(s, nullptr, &h);
+    cudaGraph_t captured = nullptr;
+    const cudaError_t ce = cudaStreamEndCapture(s->stream, &captured);
+    if (rc != CORA_OK || ce != cudaSuccess) break;
+    ok = cudaGraphInstantiate(&s->run_graph, g, 0) == cudaSuccess;
+  } while (false);
+  cudaGraphDestroy(g);
+  if (!ok) {
+    s->run_graph = nullptr;
+    cudaGetLastError();  // the fallback is the host loop; clear the sticky-free error state
+  }
+  return ok;
 }
 
 extern "C" int cora_session_reset(cora_session* s, const int32_t* prompt) {
@@ -561,6 +605,8 @@ extern "C" int cora_session_create(cora_model* m, int32_t batch, const int32_t* 
     cudaGraphDestroy(g);
     if (ce != cudaSuccess) SK(fail(CORA_ECUDA, "graph instantiate: %s", cudaGetErrorString(ce)));
   }
+  s->max_iters = int32_t(s->n_blocks) * s->T;
+  build_run_graph(s);
 #undef SK
   *out = s;
   return CORA_OK;
@@ -570,6 +616,7 @@ extern "C" int cora_session_destroy(cora_session* s) {
   if (!s) return CORA_OK;
   if (s->stream) cudaStreamSynchronize(s->stream);
   if (s->graph) cudaGraphExecDestroy(s->graph);
+  if (s->run_graph) cudaGraphExecDestroy(s->run_graph);
   for (void* p : s->allocs) cudaFree(p);
   if (s->status_h) cudaFreeHost(s->status_h);
   if (s->stream) cudaStreamDestroy(s->stream);
@@ -597,6 +644,32 @@ extern "C" int cora_denoise_step(cora_session* s, uint8_t* all_done_out) {
   const uint8_t done = reinterpret_cast<const uint8_t*>(s->status_h)[0];
   s->finished = done != 0;
   if (all_done_out) *all_done_out = done;
+  return CORA_OK;
+}
+
+extern "C" int cora_session_run(cora_session* s, int32_t* steps_out, uint8_t* on_device_out) {
+  REQUIRE(s, "cora_session_run: NULL session");
+  if (s->finished) return fail(CORA_ESTATE, "every sequence has finished; reset the session");
+  int32_t steps = 0;
+  if (s->run_graph) {
+    CK(cudaMemsetAsync(s->status + 2, 0, sizeof(int32_t), s->stream));
+    CK(cudaGraphLaunch(s->run_graph, s->stream));
+    CK(cudaMemcpyAsync(s->status_h, s->status, 3 * sizeof(int32_t), cudaMemcpyDeviceToHost, s->stream));
+    CK(cudaStreamSynchronize(s->stream));
+    steps = s->status_h[2];
+    s->batched_passes += steps;
+    if (s->status_h[1] != 0) return fail(CORA_ETIMEOUT, "device error word 0x%x after step", s->status_h[1]);
+    s->finished = reinterpret_cast<const uint8_t*>(s->status_h)[0] != 0;
+  } else {
+    uint8_t done = 0;
+    for (int32_t i = 0; i < s->max_iters && !done; ++i, ++steps) {
+      const int rc = cora_denoise_step(s, &done);
+      if (rc) return rc;
+    }
+  }
+  if (steps_out) *steps_out = steps;
+  if (on_device_out) *on_device_out = s->run_graph ? 1 : 0;
+  if (!s->finished) return fail(CORA_ESTATE, "decode did not finish within the horizon");
   return CORA_OK;
 }
 
@@ -690,13 +763,8 @@ extern "C" int cora_generate(cora_model* m, const int32_t* prompt, int32_t B, in
     rc = cora_session_reset(s, prompt);
     if (rc) return rc;
   }
-  const int64_t max_steps = int64_t(s->n_blocks) * s->T;
-  uint8_t done = 0;
-  for (int64_t i = 0; i < max_steps && !done; ++i) {
-    rc = cora_denoise_step(s, &done);
-    if (rc) return rc;
-  }
-  if (!done) return fail(CORA_ESTATE, "decode did not finish within the horizon");
+  rc = cora_session_run(s, nullptr, nullptr);
+  if (rc) return rc;
   CK(cudaMemcpy2D(tokens_out, size_t(gen_len) * 4, s->tokens + P, size_t(s->S) * 4, size_t(gen_len) * 4, B,
                   cudaMemcpyDeviceToHost));
   std::vector<int32_t> ctrl(size_t(B) * 4);

@@ -171,3 +171,36 @@ def test_batch_sequences_are_independent(tiny):
         toks1, passes1, _ = cora.cora_generate(m, prompt[b: b + 1], G, BL, T, TAU, K)
         assert passes1[0] == passes3[b]
         assert np.array_equal(toks1[0], toks3[b])
+
+
+def test_device_loop_matches_host_steps(sharp):
+    """cora_session_run (the whole decode as one graph launch with a WHILE
+    node) executes exactly the steps of a host loop over cora_denoise_step,
+    with identical results; it can run again after a reset."""
+    m, prompt = sharp
+    B = 3
+    s_dev = cora.cora_session_create(m, B, prompt, P, G, BL, T, TAU, K)
+    s_host = cora.cora_session_create(m, B, prompt, P, G, BL, T, TAU, K)
+    try:
+        steps, on_device = cora.cora_session_run(s_dev)
+        assert on_device, "the decode should run as one device-side loop"
+        host_steps, done = 0, False
+        while not done:
+            done = cora.cora_denoise_step(s_host)
+            host_steps += 1
+        assert steps == host_steps == cora.cora_session_batched_passes(s_dev)
+        a = cora.cora_session_read(s_dev, B, P + G, G, BL)
+        b = cora.cora_session_read(s_host, B, P + G, G, BL)
+        for key in ("tokens", "state", "ctrl"):
+            assert np.array_equal(a[key], b[key]), key
+        assert np.all(a["ctrl"][:, 3] == 1) and a["ctrl"][:, 2].max() == steps
+        with pytest.raises(cora.CoraError) as e:
+            cora.cora_session_run(s_dev)
+        assert e.value.code == cora.CORA_ESTATE
+        cora.cora_session_reset(s_dev, prompt)
+        steps2, _ = cora.cora_session_run(s_dev)
+        assert steps2 == steps
+        assert np.array_equal(cora.cora_session_read(s_dev, B, P + G, G, BL)["tokens"], a["tokens"])
+    finally:
+        cora.cora_session_destroy(s_dev)
+        cora.cora_session_destroy(s_host)
