@@ -364,6 +364,21 @@ def run_cora(args, cfg, ws, rank, local):
         gx = {"head_sigma": round(cfg_g["head_sigma"], 6), "tokens_per_s": round(B * G * reps / tg, 2),
               "passes_per_block": round(float(pg.mean()) / (G // BL), 3),
               "rho": round(float(pg.mean()) / ((G // BL) * T), 4), "timing": "host wall clock, e2e call"}
+        # (tau, K, schedule) sweep on the same model: the gate's operating
+        # points and the remaining-steps schedule (one warm call, one timed)
+        sweep = []
+        for tau_s, K_s, sched in ((tau, K, 0), (tau, 0, 0), (tau, 2, 0), (0.9, K, 0), (0.5, K, 0), (tau, K, 1),
+                                  (2.0, K, 0)):
+            opt = cora.decode_options(schedule=sched)
+            cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau_s, K_s, options=opt)
+            t0 = time.perf_counter()
+            _, ps, _ = cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau_s, K_s, options=opt)
+            dt = time.perf_counter() - t0
+            sweep.append({"tau": tau_s, "K": K_s, "schedule": "remaining" if sched else "fixed",
+                          "passes_per_block": round(float(ps.mean()) / (G // BL), 3),
+                          "rho": round(float(ps.mean()) / ((G // BL) * T), 4),
+                          "tokens_per_s": round(B * G / dt, 2)})
+        gx["sweep"] = sweep
         cora.cora_model_destroy(mg)
         s = None
     if s is not None:

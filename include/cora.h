@@ -61,6 +61,7 @@ extern "C" {
 #define CORA_UNRESOLVED 0  /* still masked: in U^(s) */
 #define CORA_TRANSFERRED 1 /* fixed by the original transfer rule: in T^(s) */
 #define CORA_ACCEPTED 2    /* accepted by the residual gate: in A^(s) */
+#define CORA_EOS_FILLED 3  /* set to the EOS id after a block that committed it (EOS-aware stop) */
 
 /* Returns the message of the calling thread's last failed call ("" if none). */
 CORA_API const char* cora_last_error(void);
@@ -146,6 +147,31 @@ CORA_API int cora_session_create(cora_model* m, int32_t batch, const int32_t* pr
                         int32_t block_len, int32_t steps_per_block, float tau, int32_t K, cora_session** out);
 CORA_API int cora_session_destroy(cora_session* s);
 
+/* Decoding variants: the ablations the paper discusses around Sec. 3 (its
+ * transfer schedule, where persistence starts counting, an EOS-aware stop).
+ * All-zero options but eos_id = -1 are the method as described, which is
+ * what cora_session_create uses. */
+#define CORA_SCHEDULE_FIXED 0      /* k_s from the block length: floor(BL/T), the first BL mod T steps +1 */
+#define CORA_SCHEDULE_REMAINING 1  /* k_s = ceil(|U| / (T - s)), |U| = unresolved positions of the block */
+#define CORA_PERSIST_BLOCK 0       /* Eq. 2 counters start at each block's first pass */
+#define CORA_PERSIST_CARRY 1       /* reserved: counters from a position's first pass (not yet supported) */
+typedef struct cora_decode_options {
+  int32_t schedule;     /* CORA_SCHEDULE_* */
+  int32_t persistence;  /* CORA_PERSIST_* */
+  int32_t eos_id;       /* -1: none.  Else the EOS-aware stop: once a block terminates holding this id, the
+                           sequence finishes and every later generation position takes the id
+                           (state CORA_EOS_FILLED); later blocks execute no pass.  Must be a
+                           vocabulary id other than the mask id. */
+} cora_decode_options;
+
+/* cora_session_create with decoding options (NULL = defaults).  The options
+ * are fixed for the session's lifetime (they are baked into its graphs).
+ * Errors as cora_session_create; CORA_EINVAL for an unknown or unsupported
+ * option value. */
+CORA_API int cora_session_create_ex(cora_model* m, int32_t batch, const int32_t* prompt, int32_t prompt_len,
+                                    int32_t gen_len, int32_t block_len, int32_t steps_per_block, float tau,
+                                    int32_t K, const cora_decode_options* opt, cora_session** out);
+
 /* Re-initialises the canvas from a new prompt (same shapes) and resets every
  * block/step/pass counter.  `prompt` is "any".  Synchronous. */
 CORA_API int cora_session_reset(cora_session* s, const int32_t* prompt);
@@ -173,7 +199,7 @@ CORA_API int cora_session_run(cora_session* s, int32_t* steps_out, uint8_t* on_d
 
 /* Copies session state to host buffers (any pointer may be NULL; synchronous):
  *   tokens  int32 [B, prompt_len + gen_len]   canvas
- *   state   uint8 [B, gen_len]               CORA_UNRESOLVED/TRANSFERRED/ACCEPTED
+ *   state   uint8 [B, gen_len]               CORA_UNRESOLVED/TRANSFERRED/ACCEPTED/EOS_FILLED
  *   persist int32 [B, block_len]             Eq. 2 counters of the active block
  *   prev    int32 [B, block_len]             previous executed step's x_hat (-1: none)
  *   ctrl    int32 [B, 4]                     {block, step, passes executed, finished}
@@ -231,6 +257,13 @@ CORA_API int cora_session_batched_passes(cora_session* s, int64_t* out);
 CORA_API int cora_generate(cora_model* m, const int32_t* prompt, int32_t B, int32_t P, int32_t gen_len, int32_t block_len,
                   int32_t steps_per_block, float tau, int32_t K, int32_t* tokens_out, int64_t* passes_out,
                   int64_t* batched_passes_out);
+
+/* cora_generate with decoding options (NULL = defaults; see
+ * cora_session_create_ex). */
+CORA_API int cora_generate_ex(cora_model* m, const int32_t* prompt, int32_t B, int32_t P, int32_t gen_len,
+                              int32_t block_len, int32_t steps_per_block, float tau, int32_t K,
+                              const cora_decode_options* opt, int32_t* tokens_out, int64_t* passes_out,
+                              int64_t* batched_passes_out);
 
 /* ---------------------------------------------------------------------------
  * Gate and transfer rule on device buffers (Eq. 2, transfer rule, Eq. 3,

@@ -23,6 +23,8 @@ Readings where the paper is silent (each is listed in the design notes):
     ranked by confidence (higher first, then lower position);
   * argmax ties go to the lowest vocabulary id (the paper's "deterministically
     tie-broken" top-1, Sec. 3.2);
+  * the transfer count of a step is the fixed schedule above; the
+    "remaining-steps" variant recomputes ceil(|U| / (T - s)) each step;
   * the persistence counter and previous prediction reset at block start
     (a position's first executed step is the block's first pass);
   * the counter is updated for every position unresolved when the step
@@ -42,7 +44,9 @@ from dataclasses import dataclass, field
 import numpy as np
 
 # Position states of the generation canvas (match the CUDA library's codes).
-UNRESOLVED, TRANSFERRED, ACCEPTED = 0, 1, 2
+# EOS_FILLED marks positions after a block that committed the EOS id (the
+# EOS-aware stop variant): they take the EOS id without being decoded.
+UNRESOLVED, TRANSFERRED, ACCEPTED, EOS_FILLED = 0, 1, 2, 3
 
 
 # ---------------------------------------------------------------------------
@@ -155,6 +159,14 @@ def transfer_schedule(n: int, T: int) -> list[int]:
     return [base + (1 if s < extra else 0) for s in range(T)]
 
 
+def remaining_step_count(n_unresolved: int, T: int, s: int) -> int:
+    """The 'remaining-steps' schedule variant: at step s (0-based) of a block,
+    fix ceil(|U| / (T - s)) positions, |U| the block's unresolved count when
+    the step starts.  It fixes every position by step T - 1 and equals the
+    fixed schedule when nothing is accepted and T divides the block length."""
+    return -(-int(n_unresolved) // (T - s))
+
+
 def transfer_set(conf, unresolved, k: int) -> list[int]:
     """The min(k, |U|) unresolved positions of highest confidence.
 
@@ -237,8 +249,15 @@ class DecodeTrace:
 
 
 def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
-             tau: float, K: int, record: bool = False, forward=None) -> DecodeTrace:
-    """Decode one sequence.  ``forward(tokens) -> hidden`` defaults to the oracle."""
+             tau: float, K: int, record: bool = False, forward=None, schedule: str = "fixed",
+             eos_id: int = -1) -> DecodeTrace:
+    """Decode one sequence.  ``forward(tokens) -> hidden`` defaults to the oracle.
+
+    schedule: "fixed" (the transfer schedule of the block length, the default)
+    or "remaining" (remaining_step_count on the block's unresolved count).
+    eos_id >= 0: EOS-aware stop -- once a block has terminated holding that id,
+    every later generation position takes it (state EOS_FILLED) and the later
+    blocks execute no pass (their entries in passes_per_block are 0)."""
     if forward is None:
         def forward(tok):
             return forward_hidden(cfg, w, tok)
@@ -258,7 +277,8 @@ def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
             logits = lm_logits(cfg, w, h[lo: lo + block_len])
             conf, x_hat = top1(logits)
             before = st.copy() if record else None
-            r = cora_step(st, conf, x_hat, sched[s], tau, K)
+            k = sched[s] if schedule == "fixed" else remaining_step_count(np.sum(st.state == UNRESOLVED), T, s)
+            r = cora_step(st, conf, x_hat, k, tau, K)
             x[lo: lo + block_len] = st.tokens
             gstate[b * block_len: (b + 1) * block_len] = st.state
             n_exec += 1
@@ -268,6 +288,11 @@ def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
             if r.done:
                 break
         passes.append(n_exec)
+        if eos_id >= 0 and np.any(st.tokens == eos_id):
+            x[lo + block_len:] = eos_id
+            gstate[(b + 1) * block_len:] = EOS_FILLED
+            passes.extend([0] * (gen_len // block_len - b - 1))
+            break
     return DecodeTrace(x[P:].copy(), passes, steps)
 
 

@@ -26,7 +26,10 @@ EXPORTED = [
     "cora_session_batched_passes", "cora_generate", "cora_gate_transfer", "cora_reduce_top1", "cora_reduce_gate",
     "cora_op_gemm", "cora_op_attention", "cora_op_rmsnorm", "cora_op_lm_head_top1", "cora_synth_normal_bf16",
     "cora_device_error", "cora_session_profile_step", "cora_session_stream", "cora_reduce_top1_noalloc",
+    "cora_session_create_ex", "cora_generate_ex",
 ]
+SCHEDULE_FIXED, SCHEDULE_REMAINING = 0, 1
+PERSIST_BLOCK, PERSIST_CARRY = 0, 1
 KIND_NAMES = ["embed", "rmsnorm", "gemm_qkv_rope", "attention", "gemm_o_resid", "gemm_gate_up_swiglu",
               "gemm_down_resid", "final_norm", "lm_head_top1", "gate"]
 
@@ -35,6 +38,14 @@ class CoraError(RuntimeError):
     def __init__(self, fn: str, code: int, msg: str):
         super().__init__(f"{fn} failed with status {code}: {msg}")
         self.code = code
+
+
+class DecodeOptions(C.Structure):
+    _fields_ = [("schedule", C.c_int32), ("persistence", C.c_int32), ("eos_id", C.c_int32)]
+
+
+def decode_options(schedule=SCHEDULE_FIXED, persistence=PERSIST_BLOCK, eos_id=-1) -> DecodeOptions:
+    return DecodeOptions(schedule, persistence, eos_id)
 
 
 class ModelConfig(C.Structure):
@@ -84,6 +95,8 @@ def lib():
             "cora_session_profile_step": ([vp, i32, vp, vp, vp], C.c_int),
             "cora_session_stream": ([vp, C.POINTER(vp)], C.c_int),
             "cora_generate": ([vp, vp, i32, i32, i32, i32, i32, f32, i32, vp, vp, vp], C.c_int),
+            "cora_session_create_ex": ([vp, i32, vp, i32, i32, i32, i32, f32, i32, vp, C.POINTER(vp)], C.c_int),
+            "cora_generate_ex": ([vp, vp, i32, i32, i32, i32, i32, f32, i32, vp, vp, vp, vp], C.c_int),
             "cora_gate_transfer": ([vp] * 6 + [i32, i32, i32, f32, i32] + [vp] * 3 + [vp], C.c_int),
             "cora_reduce_top1": ([vp, i32, i32, vp, vp, vp], C.c_int),
             "cora_reduce_top1_noalloc": ([vp, i32, i32, vp, vp, vp], C.c_int),
@@ -159,10 +172,16 @@ def cora_model_destroy(model: int) -> None:
     _check("cora_model_destroy", lib().cora_model_destroy(model))
 
 
-def cora_session_create(model, batch, prompt, prompt_len, gen_len, block_len, steps_per_block, tau, K) -> int:
+def cora_session_create(model, batch, prompt, prompt_len, gen_len, block_len, steps_per_block, tau, K,
+                        options: DecodeOptions | None = None) -> int:
     out = C.c_void_p()
-    _check("cora_session_create", lib().cora_session_create(model, batch, ptr(prompt), prompt_len, gen_len,
-                                                            block_len, steps_per_block, tau, K, C.byref(out)))
+    if options is None:
+        _check("cora_session_create", lib().cora_session_create(model, batch, ptr(prompt), prompt_len, gen_len,
+                                                                block_len, steps_per_block, tau, K, C.byref(out)))
+    else:
+        _check("cora_session_create_ex", lib().cora_session_create_ex(
+            model, batch, ptr(prompt), prompt_len, gen_len, block_len, steps_per_block, tau, K,
+            C.cast(C.byref(options), C.c_void_p), C.byref(out)))
     return out.value
 
 
@@ -228,7 +247,8 @@ def cora_session_batched_passes(session) -> int:
     return int(out[0])
 
 
-def cora_generate(model, prompt, gen_len, block_len, steps_per_block, tau, K):
+def cora_generate(model, prompt, gen_len, block_len, steps_per_block, tau, K,
+                  options: DecodeOptions | None = None):
     """prompt: [B, P] int32 (host numpy or device tensor).  Returns (tokens [B, G], passes [B], batched)."""
     B, P = prompt.shape
     tokens = np.zeros((B, gen_len), np.int32)
@@ -236,8 +256,13 @@ def cora_generate(model, prompt, gen_len, block_len, steps_per_block, tau, K):
     batched = np.zeros(1, np.int64)
     if isinstance(prompt, np.ndarray):
         prompt = np.ascontiguousarray(prompt, dtype=np.int32)
-    _check("cora_generate", lib().cora_generate(model, ptr(prompt), B, P, gen_len, block_len, steps_per_block,
-                                                tau, K, ptr(tokens), ptr(passes), ptr(batched)))
+    if options is None:
+        _check("cora_generate", lib().cora_generate(model, ptr(prompt), B, P, gen_len, block_len, steps_per_block,
+                                                    tau, K, ptr(tokens), ptr(passes), ptr(batched)))
+    else:
+        _check("cora_generate_ex", lib().cora_generate_ex(
+            model, ptr(prompt), B, P, gen_len, block_len, steps_per_block, tau, K,
+            C.cast(C.byref(options), C.c_void_p), ptr(tokens), ptr(passes), ptr(batched)))
     return tokens, passes, int(batched[0])
 
 

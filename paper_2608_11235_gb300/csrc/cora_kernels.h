@@ -57,6 +57,8 @@ struct SessionGateArgs {
   int B, S, P, G, BL, T;
   float tau;
   int K;
+  int schedule;  // CORA_SCHEDULE_*
+  int eos_id;    // < 0: none
 };
 
 void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_t start, float scale,

@@ -295,8 +295,15 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
       g.state = a.state[gpos];
       g.token = a.tokens[cpos];
     }
-    const int base = a.BL / a.T, extra = a.BL % a.T;
-    const int k = base + (step < extra ? 1 : 0);  // transfer schedule
+    int k;
+    if (a.schedule == CORA_SCHEDULE_REMAINING) {
+      // ceil(|U| / (T - s)) over the block's positions unresolved now
+      const int n_u = __popc(__ballot_sync(0xffffffffu, valid && g.state == CORA_UNRESOLVED));
+      k = (n_u + (a.T - step) - 1) / (a.T - step);
+    } else {
+      const int base = a.BL / a.T, extra = a.BL % a.T;
+      k = base + (step < extra ? 1 : 0);  // transfer schedule of the block length
+    }
     const bool blk_done = gate_warp(g, valid, k, a.tau, a.K);
     if (valid) {
       a.state[gpos] = static_cast<uint8_t>(g.state);
@@ -306,13 +313,23 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
       a.prev[r] = blk_done ? -1 : g.prev;      // fresh state for the next block
       a.persist[r] = blk_done ? 0 : g.persist;
     }
+    // EOS-aware stop: a terminated block holding the EOS id ends the sequence;
+    // every later generation position takes the EOS id (state EOS_FILLED).
+    const bool eos_stop =
+        blk_done && a.eos_id >= 0 && __any_sync(0xffffffffu, valid && g.token == a.eos_id) && blk + 1 < n_blocks;
+    if (eos_stop) {
+      for (int i = (blk + 1) * a.BL + lane; i < a.G; i += 32) {
+        a.tokens[static_cast<int64_t>(b) * a.S + a.P + i] = a.eos_id;
+        a.state[static_cast<int64_t>(b) * a.G + i] = CORA_EOS_FILLED;
+      }
+    }
     __syncwarp();
     if (lane == 0) {
       ctrl[2] += 1;  // executed passes of this sequence
       if (blk_done) {
         ctrl[0] = blk + 1;
         ctrl[1] = 0;
-        if (blk + 1 >= n_blocks) ctrl[3] = 1;
+        if (blk + 1 >= n_blocks || eos_stop) ctrl[3] = 1;
       } else if (step + 1 >= a.T) {
         // The schedule fixes every position by the horizon; reaching it with
         // unresolved positions is an internal error.

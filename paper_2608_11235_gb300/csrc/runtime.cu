@@ -329,6 +329,7 @@ struct cora_session {
   cora_model* m = nullptr;
   int B = 0, P = 0, G = 0, S = 0, BL = 0, T = 0, n_blocks = 0, M = 0, R = 0;
   float tau = 0.f;
+  cora_decode_options opt{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1};
   int K = 0;
   cudaStream_t stream = nullptr;
   std::vector<void*> allocs;
@@ -444,7 +445,7 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
   SessionGateArgs ga{s->parts, s->n_parts, s->ctrl,  s->tokens, s->state,  s->persist, s->prev,
                      s->conf,  s->argmax,  s->unmask, s->accept, reinterpret_cast<uint8_t*>(s->status),
                      err,      s->B,       s->S,      s->P,      s->G,       s->BL,      s->T,
-                     s->tau,   s->K};
+                     s->tau,   s->K,       s->opt.schedule, s->opt.eos_id};
   launch_session_gate(ga, st);
   REC(CORA_KIND_GATE);
   CK(cudaGetLastError());
@@ -505,7 +506,20 @@ extern "C" int cora_session_reset(cora_session* s, const int32_t* prompt) {
 extern "C" int cora_session_create(cora_model* m, int32_t batch, const int32_t* prompt, int32_t prompt_len,
                                    int32_t gen_len, int32_t block_len, int32_t steps_per_block, float tau, int32_t K,
                                    cora_session** out) {
+  return cora_session_create_ex(m, batch, prompt, prompt_len, gen_len, block_len, steps_per_block, tau, K, nullptr,
+                                out);
+}
+
+extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_t* prompt, int32_t prompt_len,
+                                      int32_t gen_len, int32_t block_len, int32_t steps_per_block, float tau,
+                                      int32_t K, const cora_decode_options* opt, cora_session** out) {
   REQUIRE(m && out, "cora_session_create: NULL argument");
+  const cora_decode_options o = opt ? *opt : cora_decode_options{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1};
+  REQUIRE(o.schedule == CORA_SCHEDULE_FIXED || o.schedule == CORA_SCHEDULE_REMAINING, "unknown schedule %d",
+          o.schedule);
+  REQUIRE(o.persistence == CORA_PERSIST_BLOCK, "persistence mode %d is not supported", o.persistence);
+  REQUIRE(o.eos_id == -1 || (o.eos_id >= 0 && o.eos_id < m->cfg.vocab && o.eos_id != m->cfg.mask_id),
+          "eos_id must be -1 or a vocabulary id other than the mask id");
   REQUIRE(batch >= 1 && prompt_len >= 0 && gen_len >= 1, "bad batch/prompt_len/gen_len");
   REQUIRE(block_len >= 1 && block_len <= 32, "block_len must be in [1, 32]");
   REQUIRE(gen_len % block_len == 0, "gen_len %% block_len != 0");
@@ -526,6 +540,7 @@ extern "C" int cora_session_create(cora_model* m, int32_t batch, const int32_t* 
   s->R = batch * block_len;
   s->tau = tau;
   s->K = K;
+  s->opt = o;
   const size_t d = c.d_model, M = s->M;
 #define SK(call)              \
   do {                        \
@@ -746,17 +761,27 @@ extern "C" int cora_session_write(cora_session* s, const int32_t* tokens, const 
 extern "C" int cora_generate(cora_model* m, const int32_t* prompt, int32_t B, int32_t P, int32_t gen_len,
                              int32_t block_len, int32_t steps_per_block, float tau, int32_t K, int32_t* tokens_out,
                              int64_t* passes_out, int64_t* batched_passes_out) {
+  return cora_generate_ex(m, prompt, B, P, gen_len, block_len, steps_per_block, tau, K, nullptr, tokens_out,
+                          passes_out, batched_passes_out);
+}
+
+extern "C" int cora_generate_ex(cora_model* m, const int32_t* prompt, int32_t B, int32_t P, int32_t gen_len,
+                                int32_t block_len, int32_t steps_per_block, float tau, int32_t K,
+                                const cora_decode_options* opt, int32_t* tokens_out, int64_t* passes_out,
+                                int64_t* batched_passes_out) {
   REQUIRE(m && tokens_out && passes_out, "cora_generate: NULL argument");
+  const cora_decode_options o = opt ? *opt : cora_decode_options{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1};
   cora_session* s = m->cached;
-  // tau and K are baked into the captured graph, so they are part of the key.
+  // tau, K and the options are baked into the captured graphs, so they are part of the key.
   if (s && (s->B != B || s->P != P || s->G != gen_len || s->BL != block_len || s->T != steps_per_block ||
-            s->tau != tau || s->K != K)) {
+            s->tau != tau || s->K != K || s->opt.schedule != o.schedule || s->opt.persistence != o.persistence ||
+            s->opt.eos_id != o.eos_id)) {
     cora_session_destroy(s);
     s = nullptr;
   }
   int rc;
   if (!s) {
-    rc = cora_session_create(m, B, prompt, P, gen_len, block_len, steps_per_block, tau, K, &s);
+    rc = cora_session_create_ex(m, B, prompt, P, gen_len, block_len, steps_per_block, tau, K, &o, &s);
     if (rc) return rc;
     m->cached = s;
   } else {

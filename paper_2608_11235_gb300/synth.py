@@ -202,6 +202,29 @@ def prompts(seed: int, batch: int, length: int, mask_id: int) -> np.ndarray:
 
 
 # ---------------------------------------------------------------------------
+# Mid-decode canvases (full-size parity at later blocks): prompt, then every
+# block before `block` committed to uniform ids on [0, mask_id), the active
+# block with each position committed with probability `frac_resolved`, and
+# the later blocks masked.  State codes: 0 unresolved, 1 transferred.
+# ---------------------------------------------------------------------------
+CANVAS_STREAM = 0x43414E56  # "CANV"
+
+
+def mid_decode_canvas(cfg: dict, seed: int, block: int, frac_resolved: float) -> tuple:
+    """(tokens int32 [P + G], state uint8 [G]) for sequence 0 of `cfg`."""
+    P, G, BL, mask_id = cfg["prompt_len"], cfg["gen_len"], cfg["block_len"], cfg["mask_id"]
+    key = stream_key(seed, CANVAS_STREAM + block)
+    prompt = prompts(cfg["prompt_seed"], 1, P, mask_id)[0]
+    ids = uniform_int(key, 0, G, mask_id)
+    pos = np.arange(G)
+    committed = pos < block * BL
+    active = (pos >= block * BL) & (pos < (block + 1) * BL)
+    committed |= active & (uniform01(key, G, G) < frac_resolved)
+    gen = np.where(committed, ids, mask_id).astype(np.int32)
+    return np.concatenate([prompt.astype(np.int32), gen]), committed.astype(np.uint8)
+
+
+# ---------------------------------------------------------------------------
 # Gate-isolation inputs: bf16 logits [B, R, V] = Gumbel(0,1) + Delta * onehot
 # (Delta ~ U[0, 12]) plus a history of prior-step argmax tensors and a mask
 # state.  The boosted target of a row is its last history id with prob 0.8,

@@ -75,3 +75,15 @@ def test_session_argument_validation(L):
     assert L.cora_session_create(16, 1, z.ctypes.data, 8, 60, 32, 32, 0.5, 1, byref(out)) == cora.CORA_EINVAL
     assert L.cora_session_create(16, 9, z.ctypes.data, 8, 64, 32, 32, 0.5, 1, byref(out)) == cora.CORA_EINVAL
     assert L.cora_session_create(16, 1, z.ctypes.data, 8, 64, 32, 0, 0.5, 1, byref(out)) == cora.CORA_EINVAL
+
+
+def test_decode_options_validation(L):
+    """Unknown or not-yet-supported decoding options are rejected before the
+    model is touched (the model handle here is a dummy)."""
+    from ctypes import byref, c_void_p
+    out = c_void_p()
+    z = np.zeros(8, np.int32)
+    for opt in (cora.decode_options(schedule=2), cora.decode_options(persistence=5),
+                cora.decode_options(eos_id=-7)):
+        rc = L.cora_session_create_ex(16, 1, z.ctypes.data, 8, 64, 32, 32, 0.5, 1, byref(opt), byref(out))
+        assert rc == cora.CORA_EINVAL, (opt.schedule, opt.persistence, opt.eos_id)

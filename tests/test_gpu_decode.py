@@ -204,3 +204,59 @@ def test_device_loop_matches_host_steps(sharp):
     finally:
         cora.cora_session_destroy(s_dev)
         cora.cora_session_destroy(s_host)
+
+
+def test_remaining_schedule_on_gpu(sharp):
+    """Decoding option CORA_SCHEDULE_REMAINING: with the gate off it gives the
+    fixed schedule's tokens (block length = horizon); with the gate on every
+    executed step transfers ceil(|U| / (T - s)) positions and accepts by the
+    rule, on the GPU's own confidences."""
+    m, prompt = sharp
+    rem = cora.decode_options(schedule=cora.SCHEDULE_REMAINING)
+    t_fix, p_fix, _ = cora.cora_generate(m, prompt[:1], G, BL, T, 2.0, 1)
+    t_rem, p_rem, _ = cora.cora_generate(m, prompt[:1], G, BL, T, 2.0, 1, options=rem)
+    assert np.array_equal(t_fix, t_rem) and np.array_equal(p_fix, p_rem)
+    s = cora.cora_session_create(m, 1, prompt[:1], P, G, BL, T, TAU, K, options=rem)
+    try:
+        per_block, done = {}, False
+        while not done:
+            before = cora.cora_session_read(s, 1, P + G, G, BL)
+            done = cora.cora_denoise_step(s)
+            out = cora.cora_session_read(s, 1, P + G, G, BL)
+            blk, step = before["ctrl"][0, 0], before["ctrl"][0, 1]
+            gstate = before["state"][0][blk * BL:(blk + 1) * BL]
+            k = O.remaining_step_count(int((gstate == 0).sum()), T, int(step))
+            assert rule_holds(gstate, before["persist"][0], before["prev"][0], out["conf"][0], out["argmax"][0], k,
+                              TAU, K, dict(unmask=out["unmask"][0], accept=out["accept"][0]))
+            per_block[blk] = per_block.get(blk, 0) + int(out["unmask"][0].sum() + out["accept"][0].sum())
+        assert all(v == BL for v in per_block.values()) and len(per_block) == G // BL
+    finally:
+        cora.cora_session_destroy(s)
+
+
+def test_eos_stop_on_gpu(sharp):
+    """Decoding option eos_id (EOS-aware stop), per sequence of a batch."""
+    m, prompt = sharp
+    B = prompt.shape[0]
+    base, p_base, _ = cora.cora_generate(m, prompt, G, BL, T, TAU, K)
+    eos = int(base[0, 0])                                   # committed by sequence 0 in its first block
+    toks, passes, batched = cora.cora_generate(m, prompt, G, BL, T, TAU, K, options=cora.decode_options(eos_id=eos))
+    s = cora.cora_session_create(m, B, prompt, P, G, BL, T, TAU, K, options=cora.decode_options(eos_id=eos))
+    try:
+        cora.cora_session_run(s)
+        st = cora.cora_session_read(s, B, P + G, G, BL)["state"]
+    finally:
+        cora.cora_session_destroy(s)
+    stopped = 0
+    for b in range(B):
+        blocks = [i for i in range(G // BL) if np.any(base[b, i * BL:(i + 1) * BL] == eos)]
+        if not blocks or blocks[0] == G // BL - 1:
+            assert np.array_equal(toks[b], base[b]) and passes[b] == p_base[b]
+            continue
+        fb = blocks[0]
+        end = (fb + 1) * BL
+        assert np.array_equal(toks[b, :end], base[b, :end])
+        assert np.all(toks[b, end:] == eos) and np.all(st[b, end:] == 3)
+        assert passes[b] < p_base[b]
+        stopped += 1
+    assert stopped >= 1 and batched == passes.max()

@@ -1,0 +1,96 @@
+"""Pins for the decoding variants (ablations of Sec. 3): the remaining-steps
+transfer schedule and the EOS-aware stop.
+
+remaining_step_count fixes ceil(|U| / (T - s)) positions at step s.  Pinned by
+its defining properties: it resolves any block within the horizon, equals the
+fixed schedule when nothing is accepted and T divides the block length, and
+the decode loop applies it step by step (recorded traces).
+"""
+
+import numpy as np
+import pytest
+
+from oracle import cora_oracle as O
+from paper_2608_11235_gb300 import synth
+
+G, T = 8, 4
+
+
+@pytest.fixture(scope="module")
+def model(micro_cfg):
+    return micro_cfg, synth.model_weights_f64(micro_cfg)
+
+
+@pytest.fixture(scope="module")
+def prompt(micro_cfg):
+    return synth.prompts(3, 1, 6, micro_cfg["mask_id"])[0]
+
+
+def test_remaining_count_values():
+    assert O.remaining_step_count(8, 4, 0) == 2
+    assert O.remaining_step_count(3, 4, 1) == 1      # after acceptances: fewer than the fixed schedule's 2
+    assert O.remaining_step_count(5, 4, 3) == 5      # the last step fixes everything left
+    assert O.remaining_step_count(0, 4, 2) == 0
+
+
+@pytest.mark.parametrize("Tn", [1, 2, 3, 4, 7])
+def test_remaining_schedule_resolves_within_horizon(Tn):
+    for n in range(0, 3 * Tn + 1):
+        rem = n
+        for s in range(Tn):
+            k = O.remaining_step_count(rem, Tn, s)
+            assert (k >= 1) == (rem > 0)
+            rem -= min(k, rem)
+        assert rem == 0
+        if n % Tn == 0:                                  # dense and divisible: the fixed schedule
+            rem, ks = n, []
+            for s in range(Tn):
+                ks.append(O.remaining_step_count(rem, Tn, s))
+                rem -= ks[-1]
+            assert ks == O.transfer_schedule(n, Tn)
+
+
+@pytest.mark.parametrize("BL", [4, 8])
+def test_remaining_equals_fixed_with_the_gate_off(model, prompt, BL):
+    cfg, w = model
+    a = O.generate(cfg, w, prompt, G, BL, T, 2.0, 1)
+    b = O.generate(cfg, w, prompt, G, BL, T, 2.0, 1, schedule="remaining")
+    assert np.array_equal(a.tokens, b.tokens) and a.passes_per_block == b.passes_per_block
+
+
+@pytest.mark.parametrize("tau,K", [(0.3, 1), (0.5, 0), (0.2, 2)])
+def test_remaining_schedule_trace(model, prompt, tau, K):
+    cfg, w = model
+    BL = 8
+    tr = O.generate(cfg, w, prompt, G, BL, T, tau, K, record=True, schedule="remaining")
+    per_block = {}
+    for s in tr.steps:
+        U0 = s["before"].state == O.UNRESOLVED
+        k = O.remaining_step_count(int(U0.sum()), T, s["step"])
+        assert sorted(s["result"].transferred) == O.transfer_set(s["conf"], U0, k)
+        per_block[s["block"]] = per_block.get(s["block"], 0) + len(s["result"].transferred) + len(s["result"].accepted)
+    assert all(v == BL for v in per_block.values())
+    assert all(1 <= p <= T for p in tr.passes_per_block)
+
+
+def test_eos_stop_after_the_block_that_commits_it(model, prompt):
+    """EOS-aware stop: with eos_id = a token the plain decode commits in
+    block b (and none earlier), the decode is identical through block b, then
+    every later position is the EOS id and the later blocks run no pass; an
+    EOS id that is never committed changes nothing."""
+    cfg, w = model
+    BL = 4
+    base = O.generate(cfg, w, prompt, G, BL, T, 0.3, 1)
+    nb = G // BL
+    first = {}
+    for b in range(nb):
+        for t in base.tokens[b * BL:(b + 1) * BL]:
+            first.setdefault(int(t), b)
+    for eos, b in sorted(first.items(), key=lambda kv: kv[1]):
+        tr = O.generate(cfg, w, prompt, G, BL, T, 0.3, 1, eos_id=eos)
+        assert np.array_equal(tr.tokens[:(b + 1) * BL], base.tokens[:(b + 1) * BL])
+        assert np.all(tr.tokens[(b + 1) * BL:] == eos)
+        assert tr.passes_per_block == base.passes_per_block[:b + 1] + [0] * (nb - b - 1)
+    unused = next(v for v in range(cfg["vocab"]) if v not in first)
+    tr = O.generate(cfg, w, prompt, G, BL, T, 0.3, 1, eos_id=unused)
+    assert np.array_equal(tr.tokens, base.tokens) and tr.passes_per_block == base.passes_per_block
