@@ -366,6 +366,9 @@ def run_cora(args, cfg, ws, rank, local):
               "rho": round(float(pg.mean()) / ((G // BL) * T), 4), "timing": "host wall clock, e2e call"}
         # (tau, K, schedule) sweep on the same model: the gate's operating
         # points and the remaining-steps schedule (one warm call, one timed)
+        # dense endpoint Y* of the same prompts (gate off), for the disagreement columns
+        sd = cora.cora_session_create(mg, B, prompt_pin.numpy(), P, G, BL, T, 2.0, K)
+        cora.cora_session_run(sd)
         sweep = []
         for tau_s, K_s, sched in ((tau, K, 0), (tau, 0, 0), (tau, 2, 0), (0.9, K, 0), (0.5, K, 0), (tau, K, 1),
                                   (2.0, K, 0)):
@@ -374,10 +377,18 @@ def run_cora(args, cfg, ws, rank, local):
             t0 = time.perf_counter()
             _, ps, _ = cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau_s, K_s, options=opt)
             dt = time.perf_counter() - t0
+            sv = cora.cora_session_create(mg, B, prompt_pin.numpy(), P, G, BL, T, tau_s, K_s, options=opt)
+            cora.cora_session_run(sv)
+            n_acc, n_ad, n_od = cora.cora_session_disagreement(sv, sd, B)
+            cora.cora_session_destroy(sv)
             sweep.append({"tau": tau_s, "K": K_s, "schedule": "remaining" if sched else "fixed",
                           "passes_per_block": round(float(ps.mean()) / (G // BL), 3),
                           "rho": round(float(ps.mean()) / ((G // BL) * T), 4),
-                          "tokens_per_s": round(B * G / dt, 2)})
+                          "tokens_per_s": round(B * G / dt, 2),
+                          "accepted_per_seq": float(n_acc.mean()),
+                          "L_acc": round(float(np.mean(n_ad / np.maximum(1, n_acc))), 4),
+                          "L_out": round(float(np.mean(n_od / G)), 4)})
+        cora.cora_session_destroy(sd)
         gx["sweep"] = sweep
         cora.cora_model_destroy(mg)
         s = None

@@ -216,6 +216,18 @@ CORA_API int cora_session_read(cora_session* s, int32_t* tokens, uint8_t* state,
 CORA_API int cora_session_write(cora_session* s, const int32_t* tokens, const uint8_t* state, const int32_t* persist,
                        const int32_t* prev, const int32_t* ctrl);
 
+/* Disagreement with the dense endpoint (Sec. 4): compares the generation
+ * canvas of session s (a CORA decode) with that of session `dense` (the same
+ * model, prompts and shapes decoded with the gate off, i.e. Y*), after both
+ * have run.  Per sequence b, host int64 [B] (out):
+ *   n_acc       positions accepted by the residual gate (state CORA_ACCEPTED)
+ *   n_acc_diff  of those, positions whose token differs from Y*
+ *   n_out_diff  generation positions whose token differs from Y*
+ * so that L^acc = n_acc_diff / max(1, n_acc) and L^out = n_out_diff / gen_len.
+ * Synchronous.  Errors: CORA_EINVAL (NULL, shapes differ), CORA_ECUDA. */
+CORA_API int cora_session_disagreement(cora_session* s, cora_session* dense, int64_t* n_acc, int64_t* n_acc_diff,
+                                       int64_t* n_out_diff);
+
 /* Launch classes reported by cora_session_profile_step. */
 #define CORA_KIND_EMBED 0
 #define CORA_KIND_RMSNORM 1

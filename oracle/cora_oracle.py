@@ -324,6 +324,21 @@ def dense_decode(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: in
 
 
 # ---------------------------------------------------------------------------
+# Disagreement with the dense endpoint (Sec. 4): accepted-token and
+# final-output disagreement of one prompt.
+# ---------------------------------------------------------------------------
+def disagreement(tokens, state, tokens_dense) -> tuple[float, float]:
+    """(L_acc, L_out) of a CORA decode against the dense endpoint Y* on the
+    same canvas: L_acc averages 1[token != Y*] over the positions the gate
+    accepted (0 when none was), L_out over every generation position."""
+    tokens, state, ref = np.asarray(tokens), np.asarray(state), np.asarray(tokens_dense)
+    acc = [i for i in range(len(tokens)) if state[i] == ACCEPTED]
+    l_acc = sum(int(tokens[i] != ref[i]) for i in acc) / max(1, len(acc))
+    l_out = sum(int(tokens[i] != ref[i]) for i in range(len(tokens))) / len(tokens)
+    return l_acc, l_out
+
+
+# ---------------------------------------------------------------------------
 # Gate-isolation path: logits -> (c, x_hat) -> one gate step, batched.
 # ---------------------------------------------------------------------------
 def persist_from_history(history: np.ndarray):

@@ -26,7 +26,7 @@ EXPORTED = [
     "cora_session_batched_passes", "cora_generate", "cora_gate_transfer", "cora_reduce_top1", "cora_reduce_gate",
     "cora_op_gemm", "cora_op_attention", "cora_op_rmsnorm", "cora_op_lm_head_top1", "cora_synth_normal_bf16",
     "cora_device_error", "cora_session_profile_step", "cora_session_stream", "cora_reduce_top1_noalloc",
-    "cora_session_create_ex", "cora_generate_ex",
+    "cora_session_create_ex", "cora_generate_ex", "cora_session_disagreement",
 ]
 SCHEDULE_FIXED, SCHEDULE_REMAINING = 0, 1
 PERSIST_BLOCK, PERSIST_CARRY = 0, 1
@@ -97,6 +97,7 @@ def lib():
             "cora_generate": ([vp, vp, i32, i32, i32, i32, i32, f32, i32, vp, vp, vp], C.c_int),
             "cora_session_create_ex": ([vp, i32, vp, i32, i32, i32, i32, f32, i32, vp, C.POINTER(vp)], C.c_int),
             "cora_generate_ex": ([vp, vp, i32, i32, i32, i32, i32, f32, i32, vp, vp, vp, vp], C.c_int),
+            "cora_session_disagreement": ([vp, vp, vp, vp, vp], C.c_int),
             "cora_gate_transfer": ([vp] * 6 + [i32, i32, i32, f32, i32] + [vp] * 3 + [vp], C.c_int),
             "cora_reduce_top1": ([vp, i32, i32, vp, vp, vp], C.c_int),
             "cora_reduce_top1_noalloc": ([vp, i32, i32, vp, vp, vp], C.c_int),
@@ -205,6 +206,13 @@ def cora_session_run(session) -> tuple:
     dev = np.zeros(1, np.uint8)
     _check("cora_session_run", lib().cora_session_run(session, ptr(steps), ptr(dev)))
     return int(steps[0]), bool(dev[0])
+
+
+def cora_session_disagreement(session, dense, B):
+    """Per-sequence (n_acc, n_acc_diff, n_out_diff) against the dense session's canvas."""
+    n = [np.zeros(B, np.int64) for _ in range(3)]
+    _check("cora_session_disagreement", lib().cora_session_disagreement(session, dense, *[ptr(a) for a in n]))
+    return tuple(n)
 
 
 def cora_session_read(session, B, S, G, BL) -> dict:

@@ -123,6 +123,10 @@ struct GemmWorkspace {
 size_t gemm_workspace_bytes(int num_sms);
 
 // Tensor-map encoder (driver entry point fetched at runtime).
+// Disagreement counts of a canvas against a reference canvas: out [B][3].
+void launch_disagreement(const int32_t* tok, const uint8_t* state, const int32_t* ref, int B, int S, int P, int G,
+                         long long* out, cudaStream_t st);
+
 // One-thread kernel that sets the WHILE condition of the whole-decode graph.
 cudaError_t launch_step_loop_cond(cudaGraphConditionalHandle h, int32_t* status, int32_t max_iters, cudaStream_t st);
 

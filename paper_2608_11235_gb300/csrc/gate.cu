@@ -348,6 +348,37 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
   }
 }
 
+// Disagreement with the dense endpoint (Sec. 4), one CTA per sequence:
+// out[b] = {positions accepted by the gate, of those the ones whose token
+// differs from the dense endpoint's, generation positions that differ}.
+__global__ void disagreement_kernel(const int32_t* __restrict__ tok, const uint8_t* __restrict__ state,
+                                    const int32_t* __restrict__ ref, int S, int P, int G, long long* out) {
+  const int b = blockIdx.x;
+  int n[3] = {0, 0, 0};
+  for (int i = threadIdx.x; i < G; i += blockDim.x) {
+    const int64_t c = static_cast<int64_t>(b) * S + P + i;
+    const bool diff = tok[c] != ref[c];
+    const bool acc = state[static_cast<int64_t>(b) * G + i] == CORA_ACCEPTED;
+    n[0] += acc;
+    n[1] += acc && diff;
+    n[2] += diff;
+  }
+  __shared__ int red[3][32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+#pragma unroll
+  for (int q = 0; q < 3; ++q) {
+    int v = n[q];
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    if (lane == 0) red[q][w] = v;
+  }
+  __syncthreads();
+  if (threadIdx.x < 3) {
+    long long t = 0;
+    for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) t += red[threadIdx.x][i];
+    out[b * 3 + threadIdx.x] = t;
+  }
+}
+
 // Loop control of the whole-decode graph (a conditional WHILE node around
 // one step): counts the pass in status[2] and keeps looping while some
 // sequence is unfinished, no kernel has recorded an error and the horizon
@@ -469,4 +500,9 @@ extern "C" int cora_reduce_top1_noalloc(const uint16_t* logits, int32_t rows, in
 cudaError_t launch_step_loop_cond(cudaGraphConditionalHandle h, int32_t* status, int32_t max_iters, cudaStream_t st) {
   step_loop_cond_kernel<<<1, 1, 0, st>>>(h, status, max_iters);
   return cudaGetLastError();
+}
+
+void launch_disagreement(const int32_t* tok, const uint8_t* state, const int32_t* ref, int B, int S, int P, int G,
+                         long long* out, cudaStream_t st) {
+  disagreement_kernel<<<B, 256, 0, st>>>(tok, state, ref, S, P, G, out);
 }

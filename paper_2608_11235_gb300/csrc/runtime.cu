@@ -354,6 +354,7 @@ struct cora_session {
   uint8_t* accept = nullptr;   // [B, BL]
   int32_t* status = nullptr;   // device {all_done (byte 0), error word}
   int32_t* status_h = nullptr; // pinned host copy
+  long long* diag = nullptr;   // [B][3] disagreement counts
   CUtensorMap tm_xn{}, tm_attn{}, tm_act{}, tm_xf{};
   CUtensorMap tmo_qkv{}, tmo_h{}, tmo_act{};  // GEMM output maps
   CUtensorMap tm_qkv_in{};                     // QKV as the attention kernel's TMA source
@@ -572,6 +573,7 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   SK(sess_alloc(s, size_t(s->R), &s->unmask));
   SK(sess_alloc(s, size_t(s->R), &s->accept));
   SK(sess_alloc(s, 4, &s->status));
+  SK(sess_alloc(s, size_t(batch) * 3, &s->diag));
   SK(sess_alloc(s, gemm_workspace_bytes(m->num_sms) / sizeof(float), &s->gemm_ws.partial));
   SK(sess_alloc(s, size_t(m->num_sms), &s->gemm_ws.flags));
   if (cudaMemset(s->gemm_ws.flags, 0, sizeof(int) * m->num_sms) != cudaSuccess) SK(fail(CORA_ECUDA, "memset"));
@@ -685,6 +687,24 @@ extern "C" int cora_session_run(cora_session* s, int32_t* steps_out, uint8_t* on
   if (steps_out) *steps_out = steps;
   if (on_device_out) *on_device_out = s->run_graph ? 1 : 0;
   if (!s->finished) return fail(CORA_ESTATE, "decode did not finish within the horizon");
+  return CORA_OK;
+}
+
+extern "C" int cora_session_disagreement(cora_session* s, cora_session* dense, int64_t* n_acc, int64_t* n_acc_diff,
+                                         int64_t* n_out_diff) {
+  REQUIRE(s && dense && n_acc && n_acc_diff && n_out_diff, "cora_session_disagreement: NULL argument");
+  REQUIRE(s->B == dense->B && s->P == dense->P && s->G == dense->G, "the sessions' shapes differ");
+  CK(cudaStreamSynchronize(dense->stream));
+  launch_disagreement(s->tokens, s->state, dense->tokens, s->B, s->S, s->P, s->G, s->diag, s->stream);
+  CK(cudaGetLastError());
+  std::vector<long long> h(size_t(s->B) * 3);
+  CK(cudaMemcpyAsync(h.data(), s->diag, h.size() * sizeof(long long), cudaMemcpyDeviceToHost, s->stream));
+  CK(cudaStreamSynchronize(s->stream));
+  for (int b = 0; b < s->B; ++b) {
+    n_acc[b] = h[size_t(b) * 3];
+    n_acc_diff[b] = h[size_t(b) * 3 + 1];
+    n_out_diff[b] = h[size_t(b) * 3 + 2];
+  }
   return CORA_OK;
 }
 

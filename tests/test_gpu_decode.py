@@ -260,3 +260,28 @@ def test_eos_stop_on_gpu(sharp):
         assert passes[b] < p_base[b]
         stopped += 1
     assert stopped >= 1 and batched == passes.max()
+
+
+def test_disagreement_counts_on_gpu(sharp):
+    """cora_session_disagreement against the definitions (Sec. 4) applied to
+    the two sessions' canvases on the host; integer counts, so exact."""
+    m, prompt = sharp
+    B = prompt.shape[0]
+    s = cora.cora_session_create(m, B, prompt, P, G, BL, T, TAU, K)
+    d = cora.cora_session_create(m, B, prompt, P, G, BL, T, 2.0, 1)     # gate off: the dense endpoint
+    try:
+        cora.cora_session_run(s)
+        cora.cora_session_run(d)
+        n_acc, n_ad, n_od = cora.cora_session_disagreement(s, d, B)
+        a = cora.cora_session_read(s, B, P + G, G, BL)
+        ref = cora.cora_session_read(d, B, P + G, G, BL)["tokens"][:, P:]
+        for b in range(B):
+            tok, st = a["tokens"][b, P:], a["state"][b]
+            l_acc, l_out = O.disagreement(tok, st, ref[b])
+            assert n_acc[b] == int((st == O.ACCEPTED).sum()) > 0
+            assert l_acc == n_ad[b] / max(1, n_acc[b]) and l_out == n_od[b] / G
+        z = cora.cora_session_disagreement(d, d, B)
+        assert all(int(v.sum()) == 0 for v in z)
+    finally:
+        cora.cora_session_destroy(s)
+        cora.cora_session_destroy(d)

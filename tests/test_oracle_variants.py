@@ -94,3 +94,22 @@ def test_eos_stop_after_the_block_that_commits_it(model, prompt):
     unused = next(v for v in range(cfg["vocab"]) if v not in first)
     tr = O.generate(cfg, w, prompt, G, BL, T, 0.3, 1, eos_id=unused)
     assert np.array_equal(tr.tokens, base.tokens) and tr.passes_per_block == base.passes_per_block
+
+
+def test_disagreement_definitions():
+    tok = np.array([5, 1, 2, 3, 9, 9])
+    ref = np.array([5, 1, 7, 3, 9, 0])
+    st = np.array([O.TRANSFERRED, O.ACCEPTED, O.ACCEPTED, O.TRANSFERRED, O.ACCEPTED, O.TRANSFERRED])
+    l_acc, l_out = O.disagreement(tok, st, ref)
+    assert l_acc == 1 / 3 and l_out == 2 / 6               # accepted 1, 2, 4: only 2 differs; 2 and 5 differ overall
+    assert O.disagreement(tok, np.zeros(6, np.uint8), ref) == (0.0, 2 / 6)   # nothing accepted: L_acc = 0
+
+
+def test_disagreement_gate_off_is_zero(model, prompt):
+    cfg, w = model
+    dense, _ = O.dense_decode(cfg, w, prompt, G, 4, T)
+    tr = O.generate(cfg, w, prompt, G, 4, T, 2.0, 1, record=True)
+    st = np.zeros(G, np.uint8)
+    for s in tr.steps:
+        st[s["block"] * 4:(s["block"] + 1) * 4] = s["after"].state
+    assert O.disagreement(tr.tokens, st, dense) == (0.0, 0.0)
