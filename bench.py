@@ -370,9 +370,9 @@ def run_cora(args, cfg, ws, rank, local):
         sd = cora.cora_session_create(mg, B, prompt_pin.numpy(), P, G, BL, T, 2.0, K)
         cora.cora_session_run(sd)
         sweep = []
-        for tau_s, K_s, sched in ((tau, K, 0), (tau, 0, 0), (tau, 2, 0), (0.9, K, 0), (0.5, K, 0), (tau, K, 1),
-                                  (2.0, K, 0)):
-            opt = cora.decode_options(schedule=sched)
+        for tau_s, K_s, sched, pers in ((tau, K, 0, 0), (tau, 0, 0, 0), (tau, 2, 0, 0), (0.9, K, 0, 0),
+                                        (0.5, K, 0, 0), (tau, K, 1, 0), (tau, K, 0, 1), (2.0, K, 0, 0)):
+            opt = cora.decode_options(schedule=sched, persistence=pers)
             cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau_s, K_s, options=opt)
             t0 = time.perf_counter()
             _, ps, _ = cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau_s, K_s, options=opt)
@@ -382,6 +382,7 @@ def run_cora(args, cfg, ws, rank, local):
             n_acc, n_ad, n_od = cora.cora_session_disagreement(sv, sd, B)
             cora.cora_session_destroy(sv)
             sweep.append({"tau": tau_s, "K": K_s, "schedule": "remaining" if sched else "fixed",
+                          "persistence": "carry" if pers else "block",
                           "passes_per_block": round(float(ps.mean()) / (G // BL), 3),
                           "rho": round(float(ps.mean()) / ((G // BL) * T), 4),
                           "tokens_per_s": round(B * G / dt, 2),

@@ -154,7 +154,9 @@ CORA_API int cora_session_destroy(cora_session* s);
 #define CORA_SCHEDULE_FIXED 0      /* k_s from the block length: floor(BL/T), the first BL mod T steps +1 */
 #define CORA_SCHEDULE_REMAINING 1  /* k_s = ceil(|U| / (T - s)), |U| = unresolved positions of the block */
 #define CORA_PERSIST_BLOCK 0       /* Eq. 2 counters start at each block's first pass */
-#define CORA_PERSIST_CARRY 1       /* reserved: counters from a position's first pass (not yet supported) */
+#define CORA_PERSIST_CARRY 1       /* counters from a position's first executed pass: every pass runs Eq. 1
+                                      on every generation row (LM head over B * gen_len rows, in chunks of
+                                      256) and updates Eq. 2 for every unresolved position */
 typedef struct cora_decode_options {
   int32_t schedule;     /* CORA_SCHEDULE_* */
   int32_t persistence;  /* CORA_PERSIST_* */
@@ -202,6 +204,8 @@ CORA_API int cora_session_run(cora_session* s, int32_t* steps_out, uint8_t* on_d
  *   state   uint8 [B, gen_len]               CORA_UNRESOLVED/TRANSFERRED/ACCEPTED/EOS_FILLED
  *   persist int32 [B, block_len]             Eq. 2 counters of the active block
  *   prev    int32 [B, block_len]             previous executed step's x_hat (-1: none)
+ *           (CORA_PERSIST_CARRY sessions: persist, prev, conf and argmax are
+ *           [B, gen_len], one entry per generation position)
  *   ctrl    int32 [B, 4]                     {block, step, passes executed, finished}
  *   conf    float [B, block_len]             last step's c_i (Eq. 1)
  *   argmax  int32 [B, block_len]             last step's x_hat_i (Eq. 1)

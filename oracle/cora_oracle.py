@@ -250,25 +250,35 @@ class DecodeTrace:
 
 def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
              tau: float, K: int, record: bool = False, forward=None, schedule: str = "fixed",
-             eos_id: int = -1) -> DecodeTrace:
+             eos_id: int = -1, persistence: str = "block") -> DecodeTrace:
     """Decode one sequence.  ``forward(tokens) -> hidden`` defaults to the oracle.
 
     schedule: "fixed" (the transfer schedule of the block length, the default)
     or "remaining" (remaining_step_count on the block's unresolved count).
     eos_id >= 0: EOS-aware stop -- once a block has terminated holding that id,
     every later generation position takes it (state EOS_FILLED) and the later
-    blocks execute no pass (their entries in passes_per_block are 0)."""
+    blocks execute no pass (their entries in passes_per_block are 0).
+    persistence: "block" (Eq. 2 counters start at each block's first pass, the
+    default) or "carry" (every executed pass computes Eq. 1 for every
+    generation position and updates the counter of every unresolved one, so
+    a position's count starts at its first executed pass and carries into its
+    block)."""
     if forward is None:
         def forward(tok):
             return forward_hidden(cfg, w, tok)
     P = len(prompt)
     x = np.concatenate([np.asarray(prompt, np.int64), np.full(gen_len, cfg["mask_id"], np.int64)])
     gstate = np.zeros(gen_len, np.uint8)      # state of every generation position
+    g_persist = np.zeros(gen_len, np.int64)   # carry mode: Eq. 2 state of every generation position
+    g_prev = np.full(gen_len, -1, np.int64)
     passes = []
     steps = []
     for b in range(gen_len // block_len):
         lo = P + b * block_len
         st = BlockState.fresh(x[lo: lo + block_len])
+        if persistence == "carry":
+            st.persist[:] = g_persist[b * block_len:(b + 1) * block_len]
+            st.prev[:] = g_prev[b * block_len:(b + 1) * block_len]
         sched = transfer_schedule(block_len, T)
         n_exec = 0
         for s in range(T):
@@ -276,11 +286,22 @@ def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
             h = forward(x)
             logits = lm_logits(cfg, w, h[lo: lo + block_len])
             conf, x_hat = top1(logits)
+            if persistence == "carry":
+                # Eq. 2 for the unresolved positions outside the active block
+                _, xh_all = top1(lm_logits(cfg, w, h[P:]))
+                for j in range(gen_len):
+                    if b * block_len <= j < (b + 1) * block_len or gstate[j] != UNRESOLVED:
+                        continue
+                    g_persist[j] = g_persist[j] + 1 if g_prev[j] == int(xh_all[j]) else 0
+                    g_prev[j] = int(xh_all[j])
             before = st.copy() if record else None
             k = sched[s] if schedule == "fixed" else remaining_step_count(np.sum(st.state == UNRESOLVED), T, s)
             r = cora_step(st, conf, x_hat, k, tau, K)
             x[lo: lo + block_len] = st.tokens
             gstate[b * block_len: (b + 1) * block_len] = st.state
+            if persistence == "carry":
+                g_persist[b * block_len:(b + 1) * block_len] = st.persist
+                g_prev[b * block_len:(b + 1) * block_len] = st.prev
             n_exec += 1
             if record:
                 steps.append(dict(block=b, step=s, canvas=canvas, gen_state=gs, passes_before=n_exec - 1,

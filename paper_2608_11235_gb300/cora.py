@@ -215,11 +215,14 @@ def cora_session_disagreement(session, dense, B):
     return tuple(n)
 
 
-def cora_session_read(session, B, S, G, BL) -> dict:
+def cora_session_read(session, B, S, G, BL, eq1_rows=None) -> dict:
+    """eq1_rows: rows of persist/prev/conf/argmax per sequence (BL, or G for a
+    carry-over persistence session)."""
+    E = BL if eq1_rows is None else eq1_rows
     out = dict(tokens=np.zeros((B, S), np.int32), state=np.zeros((B, G), np.uint8),
-               persist=np.zeros((B, BL), np.int32), prev=np.zeros((B, BL), np.int32),
-               ctrl=np.zeros((B, 4), np.int32), conf=np.zeros((B, BL), np.float32),
-               argmax=np.zeros((B, BL), np.int32), unmask=np.zeros((B, BL), np.uint8),
+               persist=np.zeros((B, E), np.int32), prev=np.zeros((B, E), np.int32),
+               ctrl=np.zeros((B, 4), np.int32), conf=np.zeros((B, E), np.float32),
+               argmax=np.zeros((B, E), np.int32), unmask=np.zeros((B, BL), np.uint8),
                accept=np.zeros((B, BL), np.uint8))
     _check("cora_session_read", lib().cora_session_read(session, *[ptr(out[k]) for k in (
         "tokens", "state", "persist", "prev", "ctrl", "conf", "argmax", "unmask", "accept")]))

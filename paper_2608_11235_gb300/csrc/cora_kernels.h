@@ -41,15 +41,15 @@ struct Top1Part {
 
 // Gate launch parameters for the session path (one warp per sequence).
 struct SessionGateArgs {
-  const Top1Part* parts;  // [n_parts][B * BL]
+  const Top1Part* parts;  // Eq. 1 partials, chunked (see rows_per_seq)
   int n_parts;
   int32_t* ctrl;          // [B][4] {block, step, passes, finished}
   int32_t* tokens;        // [B][S]
   uint8_t* state;         // [B][G]
-  int32_t* persist;       // [B][BL]
-  int32_t* prev;          // [B][BL]
-  float* conf;            // [B][BL]
-  int32_t* argmax;        // [B][BL]
+  int32_t* persist;       // [B][rows_per_seq]
+  int32_t* prev;          // [B][rows_per_seq]
+  float* conf;            // [B][rows_per_seq]
+  int32_t* argmax;        // [B][rows_per_seq]
   uint8_t* unmask;        // [B][BL]
   uint8_t* accept;        // [B][BL]
   uint8_t* all_done;      // [1]
@@ -59,6 +59,11 @@ struct SessionGateArgs {
   int K;
   int schedule;  // CORA_SCHEDULE_*
   int eos_id;    // < 0: none
+  // Eq. 1 rows: rows_per_seq per sequence (BL: the active block; G: every
+  // generation position, carry-over persistence), their partials in chunks of
+  // chunk_rows rows ([n_chunks][n_parts][chunk_rows], the last chunk shorter).
+  int rows_per_seq;
+  int chunk_rows;
 };
 
 void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_t start, float scale,
@@ -66,7 +71,7 @@ void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_
 void launch_embed(const int32_t* tokens, const uint16_t* embed, float* h, int M, int d, cudaStream_t st);
 void launch_rmsnorm(const float* x, const uint16_t* w, uint16_t* out, int M, int d, float eps, cudaStream_t st);
 void launch_final_norm_rows(const float* h, const uint16_t* w, const int32_t* ctrl, uint16_t* out, int B, int S,
-                            int P, int BL, int n_blocks, int d, float eps, cudaStream_t st);
+                            int P, int BL, int n_blocks, int d, float eps, int rows_per_seq, cudaStream_t st);
 
 // Gate buffers of B blocks of R positions ([B, R] each; done is [B]).
 struct GateBuffers {

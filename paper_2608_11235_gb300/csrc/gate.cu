@@ -267,11 +267,15 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
   const int lane = threadIdx.x & 31;
   const int nw = blockDim.x >> 5;
   const int n_blocks = a.G / a.BL;
-  const int R = a.B * a.BL;
+  const int Re = a.B * a.rows_per_seq;
+  const bool carry = a.rows_per_seq != a.BL;
   // Eq. 1: every warp combines whole rows' partials (rows of finished
   // sequences included; they are ignored below).
-  for (int r = threadIdx.x >> 5; r < R; r += nw) {
-    const Top1 st = warp_combine_parts(a.parts, a.n_parts, R, r);
+  for (int r = threadIdx.x >> 5; r < Re; r += nw) {
+    const int c = r / a.chunk_rows, lr = r - c * a.chunk_rows;
+    const int rows_c = min(a.chunk_rows, Re - c * a.chunk_rows);
+    const Top1 st =
+        warp_combine_parts(a.parts + static_cast<int64_t>(c) * a.n_parts * a.chunk_rows, a.n_parts, rows_c, lr);
     if (lane == 0) {
       a.conf[r] = 1.f / st.s;
       a.argmax[r] = st.idx;
@@ -282,8 +286,22 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
     int32_t* ctrl = a.ctrl + b * 4;
     if (ctrl[3]) continue;  // finished: nothing to do (warp-uniform)
     const int blk = ctrl[0], step = ctrl[1];
+    if (carry) {
+      // Carry-over persistence: Eq. 2 for every unresolved generation
+      // position outside the active block (the block's own are updated by
+      // the gate below).
+      for (int j = lane; j < a.G; j += 32) {
+        if (j >= blk * a.BL && j < (blk + 1) * a.BL) continue;
+        if (a.state[static_cast<int64_t>(b) * a.G + j] != CORA_UNRESOLVED) continue;
+        const int rj = b * a.G + j;
+        const int32_t xh = a.argmax[rj];
+        a.persist[rj] = a.prev[rj] == xh ? a.persist[rj] + 1 : 0;
+        a.prev[rj] = xh;
+      }
+    }
     const bool valid = lane < a.BL;
-    const int r = b * a.BL + lane;
+    const int r = b * a.rows_per_seq + (carry ? blk * a.BL : 0) + lane;  // Eq. 1 / Eq. 2 row
+    const int ru = b * a.BL + lane;                                       // T / A indicator row
     const int64_t cpos = static_cast<int64_t>(b) * a.S + a.P + static_cast<int64_t>(blk) * a.BL + lane;
     const int64_t gpos = static_cast<int64_t>(b) * a.G + static_cast<int64_t>(blk) * a.BL + lane;
     GateLane g{};
@@ -308,10 +326,10 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
     if (valid) {
       a.state[gpos] = static_cast<uint8_t>(g.state);
       a.tokens[cpos] = g.token;
-      a.unmask[r] = g.T;
-      a.accept[r] = g.A;
-      a.prev[r] = blk_done ? -1 : g.prev;      // fresh state for the next block
-      a.persist[r] = blk_done ? 0 : g.persist;
+      a.unmask[ru] = g.T;
+      a.accept[ru] = g.A;
+      a.prev[r] = blk_done && !carry ? -1 : g.prev;  // block mode: fresh state for the next block
+      a.persist[r] = blk_done && !carry ? 0 : g.persist;
     }
     // EOS-aware stop: a terminated block holding the EOS id ends the sequence;
     // every later generation position takes the EOS id (state EOS_FILLED).

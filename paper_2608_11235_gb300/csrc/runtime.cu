@@ -8,6 +8,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <algorithm>
 #include <cmath>
 #include <mutex>
 #include <string>
@@ -355,7 +356,12 @@ struct cora_session {
   int32_t* status = nullptr;   // device {all_done (byte 0), error word}
   int32_t* status_h = nullptr; // pinned host copy
   long long* diag = nullptr;   // [B][3] disagreement counts
-  CUtensorMap tm_xn{}, tm_attn{}, tm_act{}, tm_xf{};
+  CUtensorMap tm_xn{}, tm_attn{}, tm_act{};
+  // Eq. 1 rows: Re = B * rows_per_seq (rows_per_seq = BL, or G for carry-over
+  // persistence), normalised into xf and run through the LM head in chunks
+  // of chunk_rows rows, one tensor map each.
+  int rows_per_seq = 0, Re = 0, chunk_rows = 0, n_chunks = 0;
+  std::vector<CUtensorMap> tm_xf;
   CUtensorMap tmo_qkv{}, tmo_h{}, tmo_act{};  // GEMM output maps
   CUtensorMap tm_qkv_in{};                     // QKV as the attention kernel's TMA source
   GemmWorkspace gemm_ws{nullptr, nullptr};
@@ -365,6 +371,18 @@ struct cora_session {
   int64_t batched_passes = 0;
   bool finished = false;
 };
+
+// One tensor map per LM-head chunk of the normalised Eq. 1 rows.
+static bool make_xf_maps(cora_session* s, size_t d) {
+  s->tm_xf.assign(size_t(s->n_chunks), CUtensorMap{});
+  for (int ch = 0; ch < s->n_chunks; ++ch) {
+    const int rows_c = std::min(s->chunk_rows, s->Re - ch * s->chunk_rows);
+    if (!make_tmap_bf16_2d(&s->tm_xf[ch], s->xf + size_t(ch) * s->chunk_rows * d, rows_c, d, d * 2,
+                           lm_head_npad(rows_c), 64))
+      return false;
+  }
+  return true;
+}
 
 template <typename T>
 static int sess_alloc(cora_session* s, size_t count, T** out) {
@@ -439,14 +457,18 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
     REC(CORA_KIND_GEMM_DOWN);
   }
   launch_final_norm_rows(s->h, m->final_norm, s->ctrl, s->xf, s->B, s->S, s->P, s->BL, s->n_blocks, d, c.norm_eps,
-                         st);
+                         s->rows_per_seq, st);
   REC(CORA_KIND_FINAL_NORM);
-  CK(launch_lm_head_top1(m->tm_head, s->tm_xf, s->R, c.vocab, d, s->parts, s->n_parts, err, st));
-  REC(CORA_KIND_LM_HEAD);
+  for (int ch = 0; ch < s->n_chunks; ++ch) {
+    const int rows_c = std::min(s->chunk_rows, s->Re - ch * s->chunk_rows);
+    CK(launch_lm_head_top1(m->tm_head, s->tm_xf[ch], rows_c, c.vocab, d,
+                           s->parts + size_t(ch) * s->n_parts * s->chunk_rows, s->n_parts, err, st));
+    REC(CORA_KIND_LM_HEAD);
+  }
   SessionGateArgs ga{s->parts, s->n_parts, s->ctrl,  s->tokens, s->state,  s->persist, s->prev,
                      s->conf,  s->argmax,  s->unmask, s->accept, reinterpret_cast<uint8_t*>(s->status),
                      err,      s->B,       s->S,      s->P,      s->G,       s->BL,      s->T,
-                     s->tau,   s->K,       s->opt.schedule, s->opt.eos_id};
+                     s->tau,   s->K,       s->opt.schedule, s->opt.eos_id, s->rows_per_seq, s->chunk_rows};
   launch_session_gate(ga, st);
   REC(CORA_KIND_GATE);
   CK(cudaGetLastError());
@@ -496,7 +518,7 @@ extern "C" int cora_session_reset(cora_session* s, const int32_t* prompt) {
   REQUIRE(s, "cora_session_reset: NULL session");
   if (prompt && s->P > 0) CK(cudaMemcpyAsync(s->prompt, prompt, size_t(s->B) * s->P * 4, cudaMemcpyDefault, s->stream));
   launch_session_init(s->tokens, s->prompt, s->state, s->persist, s->prev, s->ctrl, s->status, s->B, s->P, s->S, s->G,
-                      s->BL, s->m->cfg.mask_id, s->stream);
+                      s->rows_per_seq, s->m->cfg.mask_id, s->stream);
   CK(cudaGetLastError());
   CK(cudaStreamSynchronize(s->stream));
   s->batched_passes = 0;
@@ -518,7 +540,8 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   const cora_decode_options o = opt ? *opt : cora_decode_options{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1};
   REQUIRE(o.schedule == CORA_SCHEDULE_FIXED || o.schedule == CORA_SCHEDULE_REMAINING, "unknown schedule %d",
           o.schedule);
-  REQUIRE(o.persistence == CORA_PERSIST_BLOCK, "persistence mode %d is not supported", o.persistence);
+  REQUIRE(o.persistence == CORA_PERSIST_BLOCK || o.persistence == CORA_PERSIST_CARRY, "unknown persistence mode %d",
+          o.persistence);
   REQUIRE(o.eos_id == -1 || (o.eos_id >= 0 && o.eos_id < m->cfg.vocab && o.eos_id != m->cfg.mask_id),
           "eos_id must be -1 or a vocabulary id other than the mask id");
   REQUIRE(batch >= 1 && prompt_len >= 0 && gen_len >= 1, "bad batch/prompt_len/gen_len");
@@ -542,6 +565,10 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   s->tau = tau;
   s->K = K;
   s->opt = o;
+  s->rows_per_seq = o.persistence == CORA_PERSIST_CARRY ? gen_len : block_len;
+  s->Re = batch * s->rows_per_seq;
+  s->chunk_rows = std::min(s->Re, 256);
+  s->n_chunks = (s->Re + s->chunk_rows - 1) / s->chunk_rows;
   const size_t d = c.d_model, M = s->M;
 #define SK(call)              \
   do {                        \
@@ -560,16 +587,16 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   SK(sess_alloc(s, M * size_t(m->n_qkv), &s->qkv));
   SK(sess_alloc(s, M * size_t(c.n_heads) * c.head_dim, &s->attn));
   SK(sess_alloc(s, M * size_t(m->f_pad), &s->act));
-  SK(sess_alloc(s, size_t(s->R) * d, &s->xf));
+  SK(sess_alloc(s, size_t(s->Re) * d, &s->xf));
   SK(sess_alloc(s, size_t(s->S) * c.head_dim, &s->rope));
   s->n_parts = lm_head_parts_count(c.vocab, m->num_sms);
-  SK(sess_alloc(s, size_t(s->n_parts) * s->R, &s->parts));
+  SK(sess_alloc(s, size_t(s->n_parts) * s->n_chunks * s->chunk_rows, &s->parts));
   SK(sess_alloc(s, size_t(batch) * 4, &s->ctrl));
   SK(sess_alloc(s, size_t(batch) * gen_len, &s->state));
-  SK(sess_alloc(s, size_t(s->R), &s->persist));
-  SK(sess_alloc(s, size_t(s->R), &s->prev));
-  SK(sess_alloc(s, size_t(s->R), &s->conf));
-  SK(sess_alloc(s, size_t(s->R), &s->argmax));
+  SK(sess_alloc(s, size_t(s->Re), &s->persist));
+  SK(sess_alloc(s, size_t(s->Re), &s->prev));
+  SK(sess_alloc(s, size_t(s->Re), &s->conf));
+  SK(sess_alloc(s, size_t(s->Re), &s->argmax));
   SK(sess_alloc(s, size_t(s->R), &s->unmask));
   SK(sess_alloc(s, size_t(s->R), &s->accept));
   SK(sess_alloc(s, 4, &s->status));
@@ -599,7 +626,7 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   bool ok = make_tmap_bf16_2d(&s->tm_xn, s->xn, M, d, d * 2, 128, 64) &&
             make_tmap_bf16_2d(&s->tm_attn, s->attn, M, hq, hq * 2, 128, 64) &&
             make_tmap_bf16_2d(&s->tm_act, s->act, M, m->f_pad, size_t(m->f_pad) * 2, 128, 64) &&
-            make_tmap_bf16_2d(&s->tm_xf, s->xf, s->R, d, d * 2, lm_head_npad(s->R), 64) &&
+            make_xf_maps(s, d) &&
             make_gemm_out_tmap(&s->tmo_qkv, s->qkv, int(M), m->n_qkv, CORA_EPI_ROPE_BF16) &&
             make_tmap_bf16_2d(&s->tm_qkv_in, s->qkv, M, size_t(m->n_qkv), size_t(m->n_qkv) * 2, 128, 64) &&
             make_gemm_out_tmap(&s->tmo_h, s->h, int(M), int(d), CORA_EPI_RESID_F32) &&
@@ -751,11 +778,11 @@ extern "C" int cora_session_read(cora_session* s, int32_t* tokens, uint8_t* stat
   CK(cudaStreamSynchronize(s->stream));
   if (tokens) CK(cudaMemcpy(tokens, s->tokens, size_t(s->M) * 4, cudaMemcpyDeviceToHost));
   if (state) CK(cudaMemcpy(state, s->state, size_t(s->B) * s->G, cudaMemcpyDeviceToHost));
-  if (persist) CK(cudaMemcpy(persist, s->persist, size_t(s->R) * 4, cudaMemcpyDeviceToHost));
-  if (prev) CK(cudaMemcpy(prev, s->prev, size_t(s->R) * 4, cudaMemcpyDeviceToHost));
+  if (persist) CK(cudaMemcpy(persist, s->persist, size_t(s->Re) * 4, cudaMemcpyDeviceToHost));
+  if (prev) CK(cudaMemcpy(prev, s->prev, size_t(s->Re) * 4, cudaMemcpyDeviceToHost));
   if (ctrl) CK(cudaMemcpy(ctrl, s->ctrl, size_t(s->B) * 16, cudaMemcpyDeviceToHost));
-  if (conf) CK(cudaMemcpy(conf, s->conf, size_t(s->R) * 4, cudaMemcpyDeviceToHost));
-  if (argmax) CK(cudaMemcpy(argmax, s->argmax, size_t(s->R) * 4, cudaMemcpyDeviceToHost));
+  if (conf) CK(cudaMemcpy(conf, s->conf, size_t(s->Re) * 4, cudaMemcpyDeviceToHost));
+  if (argmax) CK(cudaMemcpy(argmax, s->argmax, size_t(s->Re) * 4, cudaMemcpyDeviceToHost));
   if (unmask) CK(cudaMemcpy(unmask, s->unmask, size_t(s->R), cudaMemcpyDeviceToHost));
   if (accept) CK(cudaMemcpy(accept, s->accept, size_t(s->R), cudaMemcpyDeviceToHost));
   return CORA_OK;
@@ -767,8 +794,8 @@ extern "C" int cora_session_write(cora_session* s, const int32_t* tokens, const 
   CK(cudaStreamSynchronize(s->stream));
   if (tokens) CK(cudaMemcpy(s->tokens, tokens, size_t(s->M) * 4, cudaMemcpyHostToDevice));
   if (state) CK(cudaMemcpy(s->state, state, size_t(s->B) * s->G, cudaMemcpyHostToDevice));
-  if (persist) CK(cudaMemcpy(s->persist, persist, size_t(s->R) * 4, cudaMemcpyHostToDevice));
-  if (prev) CK(cudaMemcpy(s->prev, prev, size_t(s->R) * 4, cudaMemcpyHostToDevice));
+  if (persist) CK(cudaMemcpy(s->persist, persist, size_t(s->Re) * 4, cudaMemcpyHostToDevice));
+  if (prev) CK(cudaMemcpy(s->prev, prev, size_t(s->Re) * 4, cudaMemcpyHostToDevice));
   if (ctrl) {
     CK(cudaMemcpy(s->ctrl, ctrl, size_t(s->B) * 16, cudaMemcpyHostToDevice));
     bool all = true;

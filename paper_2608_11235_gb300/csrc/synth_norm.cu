@@ -140,17 +140,23 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __re
 // Final RMSNorm on the active block's rows only: row i of sequence b is canvas
 // position prompt_len + block(b) * block_len + i.  Finished sequences keep
 // their last block (their rows are computed and ignored).
+// Final RMSNorm of the rows Eq. 1 needs: rows_per_seq == BL takes each
+// sequence's active block; otherwise (rows_per_seq == G) every generation
+// position, for the carry-over persistence variant.
 __global__ void final_norm_rows_kernel(const float* __restrict__ h, const uint16_t* __restrict__ w,
                                        const int32_t* __restrict__ ctrl, uint16_t* __restrict__ out, int B, int S,
-                                       int P, int BL, int n_blocks, int d, float eps) {
+                                       int P, int BL, int n_blocks, int d, float eps, int rows_per_seq) {
   pdl_trigger();
   pdl_wait();
   const int r = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
-  if (r >= B * BL) return;
-  const int b = r / BL, i = r % BL;
-  int blk = ctrl[b * 4 + 0];
-  blk = blk < n_blocks ? blk : n_blocks - 1;
-  const int64_t src = static_cast<int64_t>(b) * S + P + static_cast<int64_t>(blk) * BL + i;
+  if (r >= B * rows_per_seq) return;
+  const int b = r / rows_per_seq, i = r % rows_per_seq;
+  int64_t src = static_cast<int64_t>(b) * S + P + i;
+  if (rows_per_seq == BL) {
+    int blk = ctrl[b * 4 + 0];
+    blk = blk < n_blocks ? blk : n_blocks - 1;
+    src += static_cast<int64_t>(blk) * BL;
+  }
   rmsnorm_row_warp(h + src * d, w, out + static_cast<int64_t>(r) * d, d, eps, threadIdx.x & 31);
 }
 
@@ -209,8 +215,8 @@ void launch_rmsnorm(const float* x, const uint16_t* w, uint16_t* out, int M, int
 }
 
 void launch_final_norm_rows(const float* h, const uint16_t* w, const int32_t* ctrl, uint16_t* out, int B, int S,
-                            int P, int BL, int n_blocks, int d, float eps, cudaStream_t st) {
-  const int R = B * BL;
+                            int P, int BL, int n_blocks, int d, float eps, int rows_per_seq, cudaStream_t st) {
+  const int R = B * rows_per_seq;
   launch_pdl(final_norm_rows_kernel, dim3((R + 7) / 8), dim3(256), 0, st, h, w, ctrl, out, B, S, P, BL, n_blocks, d,
-             eps);
+             eps, rows_per_seq);
 }

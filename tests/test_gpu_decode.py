@@ -285,3 +285,49 @@ def test_disagreement_counts_on_gpu(sharp):
     finally:
         cora.cora_session_destroy(s)
         cora.cora_session_destroy(d)
+
+
+@pytest.mark.parametrize("Kp", [0, -1])
+def test_carry_equals_block_when_persistence_cannot_matter_gpu(sharp, Kp):
+    m, prompt = sharp
+    carry = cora.decode_options(persistence=cora.PERSIST_CARRY)
+    a = cora.cora_generate(m, prompt, G, BL, T, TAU, Kp)
+    b = cora.cora_generate(m, prompt, G, BL, T, TAU, Kp, options=carry)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1])
+
+
+def test_carry_persistence_on_gpu(sharp):
+    """CORA_PERSIST_CARRY: Eq. 1 runs on every generation row; every executed
+    step updates Eq. 2 for every unresolved position (the active block through
+    the gate, which follows the rule on the carried counters), and counters
+    are never reset at a block's end."""
+    m, prompt = sharp
+    s = cora.cora_session_create(m, 1, prompt[:1], P, G, BL, T, TAU, 1,
+                                 options=cora.decode_options(persistence=cora.PERSIST_CARRY))
+    try:
+        done, first_pass_accepts = False, 0
+        while not done:
+            bf = cora.cora_session_read(s, 1, P + G, G, BL, eq1_rows=G)
+            done = cora.cora_denoise_step(s)
+            af = cora.cora_session_read(s, 1, P + G, G, BL, eq1_rows=G)
+            blk, step = bf["ctrl"][0, 0], bf["ctrl"][0, 1]
+            lo, hi = blk * BL, (blk + 1) * BL
+            st0 = bf["state"][0]
+            k = O.transfer_schedule(BL, T)[step]
+            assert rule_holds(st0[lo:hi], bf["persist"][0, lo:hi], bf["prev"][0, lo:hi], af["conf"][0, lo:hi],
+                              af["argmax"][0, lo:hi], k, TAU, 1, dict(unmask=af["unmask"][0], accept=af["accept"][0]))
+            if step == 0:
+                first_pass_accepts += int(af["accept"][0].sum())
+            out = np.ones(G, bool)
+            out[lo:hi] = False
+            U = out & (st0 == 0)
+            want = np.where(bf["prev"][0] == af["argmax"][0], bf["persist"][0] + 1, 0)
+            assert np.array_equal(af["persist"][0][U], want[U]) and np.array_equal(af["prev"][0][U], af["argmax"][0][U])
+            keep = out & (st0 != 0)
+            assert np.array_equal(af["persist"][0][keep], bf["persist"][0][keep])
+            # active block: carried, never reset
+            Ub = st0[lo:hi] == 0
+            assert np.array_equal(af["prev"][0, lo:hi][Ub], af["argmax"][0, lo:hi][Ub])
+        print(f"carry: {first_pass_accepts} positions accepted on a block's first pass")
+    finally:
+        cora.cora_session_destroy(s)

@@ -113,3 +113,37 @@ def test_disagreement_gate_off_is_zero(model, prompt):
     for s in tr.steps:
         st[s["block"] * 4:(s["block"] + 1) * 4] = s["after"].state
     assert O.disagreement(tr.tokens, st, dense) == (0.0, 0.0)
+
+
+@pytest.mark.parametrize("K", [0, -1])
+def test_carry_equals_block_when_persistence_cannot_matter(model, prompt, K):
+    """K = 0 accepts whatever the count, K = inf never accepts: the counters'
+    starting point cannot change the decode."""
+    cfg, w = model
+    a = O.generate(cfg, w, prompt, G, 4, T, 0.3, K)
+    b = O.generate(cfg, w, prompt, G, 4, T, 0.3, K, persistence="carry")
+    assert np.array_equal(a.tokens, b.tokens) and a.passes_per_block == b.passes_per_block
+
+
+@pytest.mark.parametrize("tau,K", [(0.3, 1), (0.2, 2), (0.0, 1)])
+def test_carry_counters_brute_force(model, prompt, tau, K):
+    """Carry mode: after every executed step the counter of each position of
+    the active block that was unresolved equals the trailing run length - 1 of
+    its top-1 predictions over ALL executed passes so far (recomputed here by
+    replaying the recorded canvases through the forward)."""
+    cfg, w = model
+    BL, P = 4, len(prompt)
+    tr = O.generate(cfg, w, prompt, G, BL, T, tau, K, record=True, persistence="carry")
+    hist = []
+    for s in tr.steps:
+        h = O.forward_hidden(cfg, w, s["canvas"])
+        hist.append(O.top1(O.lm_logits(cfg, w, h[P:]))[1])
+        H = np.array(hist)                                   # [passes so far, G]
+        U0 = s["before"].state == O.UNRESOLVED
+        for i in np.flatnonzero(U0):
+            j = s["block"] * BL + i
+            run = 1
+            while run < len(H) and H[-1 - run, j] == H[-1, j]:
+                run += 1
+            assert s["after"].persist[i] == run - 1, (s["block"], s["step"], i)
+    assert any(s["step"] == 0 and s["result"].accepted for s in tr.steps) or K != 1 or tau > 0.0
