@@ -125,6 +125,53 @@ def forward_hidden(cfg: dict, w: dict, tokens: np.ndarray) -> np.ndarray:
     return h
 
 
+# ---------------------------------------------------------------------------
+# Prefix-cache step (a decoding variant): rows from `lo` on are recomputed,
+# their queries attending to keys/values of the positions before `lo` kept
+# from the block's first (dense) pass.
+# ---------------------------------------------------------------------------
+def layer_forward_prefix(cfg: dict, lw: dict, h: np.ndarray, positions: np.ndarray, k_pre: np.ndarray,
+                         v_pre: np.ndarray):
+    """One pre-norm layer on rows h [n, d] at `positions`, whose queries also
+    see the given prefix keys/values [m, Hkv, hd] (after RoPE).  Returns
+    (h_out, k, v) with this layer's keys/values of the n rows."""
+    n = h.shape[0]
+    hq, hkv, hd = cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"]
+    x = rms_norm(h, lw["attn_norm"], cfg["norm_eps"])
+    q = rope((x @ lw["wq"].T).reshape(n, hq, hd), positions, cfg["rope_theta"])
+    k = rope((x @ lw["wk"].T).reshape(n, hkv, hd), positions, cfg["rope_theta"])
+    v = (x @ lw["wv"].T).reshape(n, hkv, hd)
+    o = attention(q, np.concatenate([k_pre, k]), np.concatenate([v_pre, v])).reshape(n, hq * hd)
+    h = h + o @ lw["wo"].T
+    x = rms_norm(h, lw["ffn_norm"], cfg["norm_eps"])
+    a = silu(x @ lw["w_gate"].T) * (x @ lw["w_up"].T)
+    return h + a @ lw["w_down"].T, k, v
+
+
+def forward_hidden_kv(cfg: dict, w: dict, tokens: np.ndarray):
+    """The dense pass, also returning every layer's keys/values [S, Hkv, hd]."""
+    tokens = np.asarray(tokens)
+    hkv, hd = cfg["n_kv_heads"], cfg["head_dim"]
+    empty = np.zeros((0, hkv, hd))
+    h = w["embed"][tokens].astype(np.float64)
+    cache = []
+    for lw in w["layers"]:
+        h, k, v = layer_forward_prefix(cfg, lw, h, np.arange(len(tokens)), empty, empty)
+        cache.append((k, v))
+    return h, cache
+
+
+def forward_hidden_cached(cfg: dict, w: dict, tokens: np.ndarray, cache: list, lo: int) -> np.ndarray:
+    """Residual stream of rows lo .. S-1 after the last layer, the positions
+    before lo contributing only their cached keys/values."""
+    tokens = np.asarray(tokens)
+    h = w["embed"][tokens[lo:]].astype(np.float64)
+    pos = np.arange(lo, len(tokens))
+    for lw, (kc, vc) in zip(w["layers"], cache):
+        h, _, _ = layer_forward_prefix(cfg, lw, h, pos, kc[:lo], vc[:lo])
+    return h
+
+
 def lm_logits(cfg: dict, w: dict, h_rows: np.ndarray) -> np.ndarray:
     """Logits of the given rows: final RMSNorm, then the (untied) LM head."""
     return rms_norm(h_rows, w["final_norm"], cfg["norm_eps"]) @ w["lm_head"].T
@@ -250,7 +297,7 @@ class DecodeTrace:
 
 def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
              tau: float, K: int, record: bool = False, forward=None, schedule: str = "fixed",
-             eos_id: int = -1, persistence: str = "block") -> DecodeTrace:
+             eos_id: int = -1, persistence: str = "block", cache: str = "none") -> DecodeTrace:
     """Decode one sequence.  ``forward(tokens) -> hidden`` defaults to the oracle.
 
     schedule: "fixed" (the transfer schedule of the block length, the default)
@@ -262,7 +309,11 @@ def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
     default) or "carry" (every executed pass computes Eq. 1 for every
     generation position and updates the counter of every unresolved one, so
     a position's count starts at its first executed pass and carries into its
-    block)."""
+    block).
+    cache: "none" (the dense pass at every step, the default) or "prefix"
+    (a block's first pass is dense and keeps every layer's keys/values; its
+    later passes recompute only the rows from the active block on, see
+    forward_hidden_cached).  Not combined with carry-over persistence."""
     if forward is None:
         def forward(tok):
             return forward_hidden(cfg, w, tok)
@@ -281,9 +332,17 @@ def generate(cfg: dict, w: dict, prompt, gen_len: int, block_len: int, T: int,
             st.prev[:] = g_prev[b * block_len:(b + 1) * block_len]
         sched = transfer_schedule(block_len, T)
         n_exec = 0
+        kv = None
         for s in range(T):
             canvas, gs = (x.copy(), gstate.copy()) if record else (None, None)
-            h = forward(x)
+            if cache == "prefix":
+                if kv is None:
+                    h, kv = forward_hidden_kv(cfg, w, x)
+                else:
+                    h = np.zeros((len(x), cfg["d_model"]))
+                    h[lo:] = forward_hidden_cached(cfg, w, x, kv, lo)
+            else:
+                h = forward(x)
             logits = lm_logits(cfg, w, h[lo: lo + block_len])
             conf, x_hat = top1(logits)
             if persistence == "carry":

@@ -147,3 +147,47 @@ def test_carry_counters_brute_force(model, prompt, tau, K):
                 run += 1
             assert s["after"].persist[i] == run - 1, (s["block"], s["step"], i)
     assert any(s["step"] == 0 and s["result"].accepted for s in tr.steps) or K != 1 or tau > 0.0
+
+
+def test_prefix_layer_with_empty_prefix_is_the_dense_layer(model):
+    cfg, w = model
+    rng = np.random.default_rng(0)
+    h = rng.normal(size=(7, cfg["d_model"]))
+    e = np.zeros((0, cfg["n_kv_heads"], cfg["head_dim"]))
+    out, _, _ = O.layer_forward_prefix(cfg, w["layers"][0], h, np.arange(7), e, e)
+    assert np.allclose(out, O.layer_forward(cfg, w["layers"][0], h, np.arange(7)), rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("lo", [0, 3, 6, 13])
+def test_cache_of_the_same_canvas_reproduces_the_dense_rows(model, prompt, lo):
+    """Keys/values cached from a canvas, reused for that same canvas, give the
+    dense pass's rows exactly (the approximation only enters once the canvas
+    changes after the cache was taken)."""
+    cfg, w = model
+    x = np.concatenate([prompt, np.full(G, cfg["mask_id"])])
+    x[8:10] = [2, 5]
+    h_dense = O.forward_hidden(cfg, w, x)
+    h_kv, cache = O.forward_hidden_kv(cfg, w, x)
+    assert np.allclose(h_kv, h_dense, rtol=0, atol=1e-12)
+    assert np.allclose(O.forward_hidden_cached(cfg, w, x, cache, lo), h_dense[lo:], rtol=0, atol=1e-12)
+
+
+def test_prefix_cache_decode(model, prompt):
+    """Cached decode: every block's first pass is the dense pass of its canvas;
+    with no prompt and a single block every pass recomputes every row, so the
+    decode equals the uncached one; trace invariants hold."""
+    cfg, w = model
+    BL = 4
+    tr = O.generate(cfg, w, prompt, G, BL, T, 0.3, 1, record=True, cache="prefix")
+    for s in tr.steps:
+        if s["step"] == 0:
+            lo = len(prompt) + s["block"] * BL
+            ref = O.lm_logits(cfg, w, O.forward_hidden(cfg, w, s["canvas"])[lo: lo + BL])
+            assert np.allclose(s["logits"], ref, rtol=0, atol=1e-10)
+    per_block = {}
+    for s in tr.steps:
+        per_block[s["block"]] = per_block.get(s["block"], 0) + len(s["result"].transferred) + len(s["result"].accepted)
+    assert all(v == BL for v in per_block.values())
+    a = O.generate(cfg, w, prompt[:0], 8, 8, T, 0.3, 1)
+    b = O.generate(cfg, w, prompt[:0], 8, 8, T, 0.3, 1, cache="prefix")
+    assert np.array_equal(a.tokens, b.tokens) and a.passes_per_block == b.passes_per_block
