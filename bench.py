@@ -297,6 +297,30 @@ def run_cora(args, cfg, ws, rank, local):
     out = cora.cora_session_read(s, B, P + G, G, BL)
     per_seq_passes = out["ctrl"][:, 2].astype(float)
 
+    # ----- the same decode with the prefix cache (decoding variant): a block's
+    # first pass dense, its later passes over the rows from the active block on
+    pc = None
+    if not args.no_variant and BL == 32:
+        sc = cora.cora_session_create(m, B, prompt_dev, P, G, BL, T, tau, K,
+                                      options=cora.decode_options(cache=cora.CACHE_PREFIX))
+        stc = torch.cuda.ExternalStream(cora.cora_session_stream(sc))
+        cora.cora_session_reset(sc, prompt_dev)
+        cora.cora_session_run(sc)
+        reps = max(1, min(args.steps, 3))
+        q0, q1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        q0.record(stc)
+        steps_c = 0
+        for _ in range(reps):
+            cora.cora_session_reset(sc, prompt_dev)
+            steps_c += cora.cora_session_run(sc)[0]
+        q1.record(stc)
+        q1.synchronize()
+        ms_c = q0.elapsed_time(q1) / reps
+        cora.cora_session_destroy(sc)
+        pc = {"tokens_per_s": round(B * G / (ms_c * 1e-3), 3), "ms_per_decode": round(ms_c, 3),
+              "passes": steps_c // reps, "dense_passes": G // BL, "cached_passes": steps_c // reps - G // BL,
+              "timing": "CUDA events on the session stream, device-resident prompt"}
+
     # ----- per-kernel device times (one eager pass with events around each launch)
     cora.cora_session_reset(s, prompt_dev)
     prof = cora.cora_session_profile_step(s, cfg["n_layers"])
@@ -424,6 +448,7 @@ def run_cora(args, cfg, ws, rank, local):
         "gpu_launches": int(total_passes * launches_per_pass + args.steps),
         "clocks": clocks,
         "gate_exercising": gx,
+        "prefix_cache": pc,
         "gate_isolation": gate_iso,
     }
     return result, float(per_seq_passes.mean())

@@ -150,13 +150,22 @@ CORA_API int cora_session_destroy(cora_session* s);
 /* Decoding variants: the ablations the paper discusses around Sec. 3 (its
  * transfer schedule, where persistence starts counting, an EOS-aware stop).
  * All-zero options but eos_id = -1 are the method as described, which is
- * what cora_session_create uses. */
+ * what cora_session_create uses.  Prefix-cache sessions run cora_session_run
+ * as a host loop (one graph per block). */
 #define CORA_SCHEDULE_FIXED 0      /* k_s from the block length: floor(BL/T), the first BL mod T steps +1 */
 #define CORA_SCHEDULE_REMAINING 1  /* k_s = ceil(|U| / (T - s)), |U| = unresolved positions of the block */
 #define CORA_PERSIST_BLOCK 0       /* Eq. 2 counters start at each block's first pass */
 #define CORA_PERSIST_CARRY 1       /* counters from a position's first executed pass: every pass runs Eq. 1
                                       on every generation row (LM head over B * gen_len rows, in chunks of
                                       256) and updates Eq. 2 for every unresolved position */
+#define CORA_CACHE_NONE 0          /* the dense pass at every executed step (Sec. 3) */
+#define CORA_CACHE_PREFIX 1        /* a block's first pass is dense and keeps every layer's keys/values; its
+                                      later passes recompute only the rows from the active block to the end
+                                      of the canvas, attending to the kept keys/values of earlier positions.
+                                      The sequences of a batch then move to the next block together (a
+                                      sequence whose block ended waits; its own passes and tokens are those
+                                      of a batch of one).  Not combined with CORA_PERSIST_CARRY;
+                                      needs block_len == 32. */
 typedef struct cora_decode_options {
   int32_t schedule;     /* CORA_SCHEDULE_* */
   int32_t persistence;  /* CORA_PERSIST_* */
@@ -164,6 +173,7 @@ typedef struct cora_decode_options {
                            sequence finishes and every later generation position takes the id
                            (state CORA_EOS_FILLED); later blocks execute no pass.  Must be a
                            vocabulary id other than the mask id. */
+  int32_t cache;        /* CORA_CACHE_* */
 } cora_decode_options;
 
 /* cora_session_create with decoding options (NULL = defaults).  The options
@@ -216,7 +226,10 @@ CORA_API int cora_session_read(cora_session* s, int32_t* tokens, uint8_t* state,
 
 /* Overwrites session state from host buffers (same layouts as
  * cora_session_read; NULL leaves a part unchanged).  Lets a caller resume a
- * decode at block/step granularity.  Synchronous. */
+ * decode at block/step granularity.  In a prefix-cache session, writing ctrl
+ * at a block's step 0 (or at another block than the current one) makes the
+ * next pass that block's dense first pass; a later step of the current block
+ * keeps the keys/values its first pass kept.  Synchronous. */
 CORA_API int cora_session_write(cora_session* s, const int32_t* tokens, const uint8_t* state, const int32_t* persist,
                        const int32_t* prev, const int32_t* ctrl);
 

@@ -30,6 +30,7 @@ EXPORTED = [
 ]
 SCHEDULE_FIXED, SCHEDULE_REMAINING = 0, 1
 PERSIST_BLOCK, PERSIST_CARRY = 0, 1
+CACHE_NONE, CACHE_PREFIX = 0, 1
 KIND_NAMES = ["embed", "rmsnorm", "gemm_qkv_rope", "attention", "gemm_o_resid", "gemm_gate_up_swiglu",
               "gemm_down_resid", "final_norm", "lm_head_top1", "gate"]
 
@@ -41,11 +42,11 @@ class CoraError(RuntimeError):
 
 
 class DecodeOptions(C.Structure):
-    _fields_ = [("schedule", C.c_int32), ("persistence", C.c_int32), ("eos_id", C.c_int32)]
+    _fields_ = [("schedule", C.c_int32), ("persistence", C.c_int32), ("eos_id", C.c_int32), ("cache", C.c_int32)]
 
 
-def decode_options(schedule=SCHEDULE_FIXED, persistence=PERSIST_BLOCK, eos_id=-1) -> DecodeOptions:
-    return DecodeOptions(schedule, persistence, eos_id)
+def decode_options(schedule=SCHEDULE_FIXED, persistence=PERSIST_BLOCK, eos_id=-1, cache=0) -> DecodeOptions:
+    return DecodeOptions(schedule, persistence, eos_id, cache)
 
 
 class ModelConfig(C.Structure):

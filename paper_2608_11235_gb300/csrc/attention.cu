@@ -63,8 +63,10 @@ __device__ __forceinline__ void load_tile(uint32_t sbase, const uint16_t* g, int
 }
 
 template <int HD>
+// Queries q_start .. q_start + q_len - 1 of each sequence (all S keys); the
+// output row of query q is (q - q_start) of the sequence's q_len rows.
 __global__ void __launch_bounds__(128) attention_kernel(const uint16_t* __restrict__ qkv, uint16_t* __restrict__ out,
-                                                        int S, int Hq, int Hkv) {
+                                                        int S, int Hq, int Hkv, int q_start, int q_len) {
   extern __shared__ __align__(128) uint16_t att_smem[];
   uint16_t* sQ = att_smem;                   // [64][HD]
   uint16_t* sK0 = sQ + kQT * HD;             // 2 x [64][HD]
@@ -78,7 +80,8 @@ __global__ void __launch_bounds__(128) attention_kernel(const uint16_t* __restri
   const uint16_t* gQ = base + static_cast<int64_t>(h) * HD;
   const uint16_t* gK = base + static_cast<int64_t>(Hq + kvh) * HD;
   const uint16_t* gV = base + static_cast<int64_t>(Hq + Hkv + kvh) * HD;
-  const int q0 = qt * kQT;
+  const int q0 = q_start + qt * kQT;
+  const int q_end = q_start + q_len;
   const int n_kt = (S + kKT - 1) / kKT;
 
   pdl_trigger();
@@ -205,12 +208,12 @@ __global__ void __launch_bounds__(128) attention_kernel(const uint16_t* __restri
   const int g = lane >> 2, t = lane & 3;
   const int r0 = q0 + warp * 16 + g, r1 = r0 + 8;
   const int64_t ldo = static_cast<int64_t>(Hq) * HD;
-  uint16_t* ob = out + static_cast<int64_t>(b) * S * ldo + static_cast<int64_t>(h) * HD;
+  uint16_t* ob = out + (static_cast<int64_t>(b) * q_len - q_start) * ldo + static_cast<int64_t>(h) * HD;
 #pragma unroll
   for (int i = 0; i < HD / 8; ++i) {
     const int col = i * 8 + t * 2;
-    if (r0 < S) *reinterpret_cast<uint32_t*>(ob + static_cast<int64_t>(r0) * ldo + col) = pack_bf16x2(o[i][0] * inv0, o[i][1] * inv0);
-    if (r1 < S) *reinterpret_cast<uint32_t*>(ob + static_cast<int64_t>(r1) * ldo + col) = pack_bf16x2(o[i][2] * inv1, o[i][3] * inv1);
+    if (r0 < q_end) *reinterpret_cast<uint32_t*>(ob + static_cast<int64_t>(r0) * ldo + col) = pack_bf16x2(o[i][0] * inv0, o[i][1] * inv0);
+    if (r1 < q_end) *reinterpret_cast<uint32_t*>(ob + static_cast<int64_t>(r1) * ldo + col) = pack_bf16x2(o[i][2] * inv1, o[i][3] * inv1);
   }
 }
 
@@ -218,13 +221,14 @@ __global__ void __launch_bounds__(128) attention_kernel(const uint16_t* __restri
 
 using namespace cora;
 
-void launch_attention(const uint16_t* qkv, uint16_t* out, int B, int S, int Hq, int Hkv, int hd, cudaStream_t st) {
-  dim3 grid((S + kQT - 1) / kQT, Hq, B);
+void launch_attention(const uint16_t* qkv, uint16_t* out, int B, int S, int Hq, int Hkv, int hd, int q_start,
+                      int q_len, cudaStream_t st) {
+  dim3 grid((q_len + kQT - 1) / kQT, Hq, B);
   const int smem = (kQT + 4 * kKT) * hd * 2;
   if (hd == 128)
-    launch_pdl(attention_kernel<128>, grid, dim3(128), smem, st, qkv, out, S, Hq, Hkv);
+    launch_pdl(attention_kernel<128>, grid, dim3(128), smem, st, qkv, out, S, Hq, Hkv, q_start, q_len);
   else
-    launch_pdl(attention_kernel<64>, grid, dim3(128), smem, st, qkv, out, S, Hq, Hkv);
+    launch_pdl(attention_kernel<64>, grid, dim3(128), smem, st, qkv, out, S, Hq, Hkv, q_start, q_len);
 }
 
 cudaError_t attention_prepare() {

@@ -98,7 +98,7 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void*
 
 __global__ void __launch_bounds__(192, 1)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ CUtensorMap tmOut, int S,
-                        int Hq, int Hkv, int* err) {
+                        int Hq, int Hkv, int q_start, int* err) {
   using namespace attn;
   // idesc: M = 128, N = 128, bf16 x bf16 -> f32; PV reads B (V) MN-major.
   constexpr uint32_t IDESC_QK = idesc_bf16_f32(128, 128);
@@ -124,7 +124,7 @@ __global__ void __launch_bounds__(192, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int kvh = h / (Hq / Hkv);
-  const int q0 = qt * QT;
+  const int q0 = q_start + qt * QT;  // queries q_start .. ; output rows relative to q_start
   const int row_base = b * S;                       // first row of this sequence in [B*S, .]
   const int n_kt = (S + KT - 1) / KT;
   const int qcol = h * HD, kcol = (Hq + kvh) * HD, vcol = (Hq + Hkv + kvh) * HD;
@@ -316,7 +316,7 @@ __global__ void __launch_bounds__(192, 1)
       __syncwarp();
       if (lane == 0) {
         for (int c = 0; c < 2; ++c)
-          tma_store_3d(&tmOut, stg + c * (OPND / 2) + sub * 32 * 128, qcol + c * 64, q0 + sub * 32, b);
+          tma_store_3d(&tmOut, stg + c * (OPND / 2) + sub * 32 * 128, qcol + c * 64, qt * QT + sub * 32, b);
         asm volatile("cp.async.bulk.commit_group;" ::: "memory");
         asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
       }
@@ -343,15 +343,15 @@ cudaError_t attention_tc_prepare() {
   return cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, attn::SMEM);
 }
 
-cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int* err,
-                                cudaStream_t st) {
-  // Output map [B][S][Hq*hd] bf16, boxes of 32 rows x 64 columns (one warp's
-  // rows, one 128-byte swizzle column).
+cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
+                                int q_len, int* err, cudaStream_t st) {
+  // Output map [B][q_len][Hq*hd] bf16, boxes of 32 rows x 64 columns (one
+  // warp's rows, one 128-byte swizzle column).
   CUtensorMap tmOut;
-  if (!make_tmap_bf16_3d(&tmOut, out, static_cast<uint64_t>(Hq) * attn::HD, S, B,
-                         static_cast<uint64_t>(Hq) * attn::HD * 2, static_cast<uint64_t>(S) * Hq * attn::HD * 2, 64,
-                         32, 1))
+  if (!make_tmap_bf16_3d(&tmOut, out, static_cast<uint64_t>(Hq) * attn::HD, q_len, B,
+                         static_cast<uint64_t>(Hq) * attn::HD * 2, static_cast<uint64_t>(q_len) * Hq * attn::HD * 2,
+                         64, 32, 1))
     return cudaErrorInvalidValue;
-  dim3 grid((S + attn::QT - 1) / attn::QT, Hq, B);
-  return launch_pdl(attention_tc_kernel, grid, dim3(192), attn::SMEM, st, tmQKV, tmOut, S, Hq, Hkv, err);
+  dim3 grid((q_len + attn::QT - 1) / attn::QT, Hq, B);
+  return launch_pdl(attention_tc_kernel, grid, dim3(192), attn::SMEM, st, tmQKV, tmOut, S, Hq, Hkv, q_start, err);
 }

@@ -64,11 +64,16 @@ struct SessionGateArgs {
   // chunk_rows rows ([n_chunks][n_parts][chunk_rows], the last chunk shorter).
   int rows_per_seq;
   int chunk_rows;
+  // Prefix-cache mode: sequences move to the next block together (a sequence
+  // whose block has ended waits, ctrl step = -1); the kernel publishes the
+  // next pass in status[3] (bit 0: a block's first, dense pass; bits 1..: block).
+  int lockstep;
 };
 
 void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_t start, float scale,
                               cudaStream_t st);
-void launch_embed(const int32_t* tokens, const uint16_t* embed, float* h, int M, int d, cudaStream_t st);
+void launch_embed(const int32_t* tokens, const uint16_t* embed, float* h, int M, int d, int S_tok, int lo,
+                  int rows_per_seq, cudaStream_t st);
 void launch_rmsnorm(const float* x, const uint16_t* w, uint16_t* out, int M, int d, float eps, cudaStream_t st);
 void launch_final_norm_rows(const float* h, const uint16_t* w, const int32_t* ctrl, uint16_t* out, int B, int S,
                             int P, int BL, int n_blocks, int d, float eps, int rows_per_seq, cudaStream_t st);
@@ -117,6 +122,11 @@ struct GemmEpilogue {
   int splits;
   int split_skew;
   int split_pair;  // 1: two k-pieces per tile, each finalising half of the columns
+  // ROPE epilogue on packed prefix-cache rows: row r is position
+  // rope_pos0 + r % seq of sequence r / seq; with out3d, C is a 3-D map
+  // [sequence][position][column] and row r is stored at that position.
+  int rope_pos0;
+  int out3d;
 };
 
 // Stream-K workspace: one fp32 partial slot of 128 x 256 per CTA plus one
@@ -163,12 +173,15 @@ cudaError_t lm_head_prepare();
 cudaError_t attention_prepare();
 cudaError_t attention_tc_prepare();
 // tcgen05 attention for head_dim 128; tmQKV: bf16 [B*S, (Hq+2Hkv)*128], box 128 rows x 64 cols.
-cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int* err,
-                                cudaStream_t st);
+cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
+                                int q_len, int* err, cudaStream_t st);
 
 void launch_session_init(int32_t* tokens, const int32_t* prompt, uint8_t* state, int32_t* persist, int32_t* prev,
                          int32_t* ctrl, int32_t* status, int B, int P, int S, int G, int BL, int mask_id,
                          cudaStream_t st);
 
 // Attention.
-void launch_attention(const uint16_t* qkv, uint16_t* out, int B, int S, int Hq, int Hkv, int hd, cudaStream_t st);
+// Queries q_start .. q_start + q_len - 1 of every sequence against all S keys;
+// out holds q_len rows per sequence.  (0, S): the dense pass.
+void launch_attention(const uint16_t* qkv, uint16_t* out, int B, int S, int Hq, int Hkv, int hd, int q_start,
+                      int q_len, cudaStream_t st);

@@ -284,7 +284,8 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
   __syncthreads();
   for (int b = threadIdx.x >> 5; b < a.B; b += nw) {
     int32_t* ctrl = a.ctrl + b * 4;
-    if (ctrl[3]) continue;  // finished: nothing to do (warp-uniform)
+    if (ctrl[3]) continue;                   // finished: nothing to do (warp-uniform)
+    if (a.lockstep && ctrl[1] < 0) continue;  // block ended, waiting for the other sequences
     const int blk = ctrl[0], step = ctrl[1];
     if (carry) {
       // Carry-over persistence: Eq. 2 for every unresolved generation
@@ -344,7 +345,9 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
     __syncwarp();
     if (lane == 0) {
       ctrl[2] += 1;  // executed passes of this sequence
-      if (blk_done) {
+      if (blk_done && a.lockstep && !eos_stop && blk + 1 < n_blocks) {
+        ctrl[1] = -1;  // wait: the sequences move to the next block together
+      } else if (blk_done) {
         ctrl[0] = blk + 1;
         ctrl[1] = 0;
         if (blk + 1 >= n_blocks || eos_stop) ctrl[3] = 1;
@@ -359,6 +362,34 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
     }
   }
   __syncthreads();
+  if (threadIdx.x == 0 && a.lockstep) {
+    // Once no unfinished sequence is still working on the block, all move on;
+    // the next pass is then the new block's first (dense) pass.
+    bool active = false, waiting = false;
+    int blk = 0;
+    for (int b = 0; b < a.B; ++b) {
+      const int32_t* c = a.ctrl + b * 4;
+      if (c[3]) continue;
+      blk = c[0];
+      if (c[1] < 0)
+        waiting = true;
+      else
+        active = true;
+    }
+    int dense_next = 0;
+    if (waiting && !active) {
+      for (int b = 0; b < a.B; ++b) {
+        int32_t* c = a.ctrl + b * 4;
+        if (!c[3] && c[1] < 0) {
+          c[0] += 1;
+          c[1] = 0;
+        }
+      }
+      blk += 1;
+      dense_next = 1;
+    }
+    reinterpret_cast<int32_t*>(a.all_done)[3] = dense_next | (blk << 1);
+  }
   if (threadIdx.x == 0) {
     uint8_t all = 1;
     for (int b = 0; b < a.B; ++b) all &= static_cast<uint8_t>(a.ctrl[b * 4 + 3] != 0);

@@ -286,14 +286,24 @@ __device__ __forceinline__ void stage_f32x16(uint8_t* unit, int lane, int j0, co
                            __float_as_uint(v[4 * q + 3])));
 }
 
-// Make the warp's staged unit visible to the async proxy and issue it.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void* src, int c0, int c1, int c2) {
+  asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2)
+               : "memory");
+}
+
+// Make the warp's staged unit visible to the async proxy and issue it
+// (c2 >= 0: a 3-D store at {c0, c1, c2}).
 __device__ __forceinline__ void stage_issue(const Stager& sg, const CUtensorMap* map, const uint8_t* unit, int c0,
-                                            int c1, bool reduce) {
+                                            int c1, bool reduce, int c2 = -1) {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   __syncwarp();
   if (sg.lane == 0) {
     if (reduce)
       tma_reduce_add_2d(map, unit, c0, c1);
+    else if (c2 >= 0)
+      tma_store_3d(map, unit, c0, c1, c2);
     else
       tma_store_2d(map, unit, c0, c1);
     bulk_commit();
@@ -357,7 +367,9 @@ __device__ __forceinline__ void gemm_epilogue_warp(const GemmEpilogue& ep, const
     }
   } else {  // CORA_EPI_ROPE_BF16: rotate pairs (j, j + hd/2) of every head
     const int hd = ep.head_dim, half = hd / 2;
-    const int pos = row0 + lane >= 0 ? (row0 + lane) % ep.seq : 0;
+    const int pos = ep.rope_pos0 + (row0 + lane >= 0 ? (row0 + lane) % ep.seq : 0);
+    // store coordinates of the warp's 32-row box (they never straddle a sequence: seq % 32 == 0 when out3d)
+    const int srow = ep.out3d ? ep.rope_pos0 + row0 % ep.seq : row0, sseq = ep.out3d ? row0 / ep.seq : -1;
     const float2* tab = reinterpret_cast<const float2*>(ep.rope) + static_cast<int64_t>(pos) * half;
 #pragma unroll 1
     for (int h0 = 0; h0 < BN; h0 += hd) {
@@ -400,10 +412,10 @@ __device__ __forceinline__ void gemm_epilogue_warp(const GemmEpilogue& ep, const
         stage_bf16x16(u2, lane, k2 + 2, v[3]);
       }
       if (hd == 128) {
-        stage_issue(sg, tmC, u1, n0 + h0, row0, false);
-        stage_issue(sg, tmC, u2, n0 + h0 + half, row0, false);
+        stage_issue(sg, tmC, u1, n0 + h0, srow, false, sseq);
+        stage_issue(sg, tmC, u2, n0 + h0 + half, srow, false, sseq);
       } else {
-        stage_issue(sg, tmC, u1, n0 + h0, row0, false);
+        stage_issue(sg, tmC, u1, n0 + h0, srow, false, sseq);
       }
     }
   }

@@ -330,7 +330,7 @@ struct cora_session {
   cora_model* m = nullptr;
   int B = 0, P = 0, G = 0, S = 0, BL = 0, T = 0, n_blocks = 0, M = 0, R = 0;
   float tau = 0.f;
-  cora_decode_options opt{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1};
+  cora_decode_options opt{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1, CORA_CACHE_NONE};
   int K = 0;
   cudaStream_t stream = nullptr;
   std::vector<void*> allocs;
@@ -365,6 +365,13 @@ struct cora_session {
   CUtensorMap tmo_qkv{}, tmo_h{}, tmo_act{};  // GEMM output maps
   CUtensorMap tm_qkv_in{};                     // QKV as the attention kernel's TMA source
   GemmWorkspace gemm_ws{nullptr, nullptr};
+  // Prefix-cache mode: per-layer QKV buffers hold every layer's keys/values
+  // (written in full by a block's dense first pass, on the recomputed rows by
+  // its later passes); one graph per block for the later passes.
+  std::vector<uint16_t*> qkv_l;
+  std::vector<CUtensorMap> tmo_qkv_l, tm_qkv_in_l, tmo_qkv3_l;
+  std::vector<cudaGraphExec_t> cgraph;
+  int32_t next_info = 1;                // status[3] of the last step: bit 0 dense pass next, bits 1.. block
   cudaGraphExec_t graph = nullptr;      // one step
   cudaGraphExec_t run_graph = nullptr;  // WHILE node around one step: a whole decode (null: not available)
   int32_t max_iters = 0;                // n_blocks * T
@@ -419,29 +426,41 @@ struct LaunchRecorder {
 // whole-decode WHILE node: the status read-back is replaced by the kernel
 // that sets the loop condition.
 static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
-                        const cudaGraphConditionalHandle* loop = nullptr) {
+                        const cudaGraphConditionalHandle* loop = nullptr, int cached_block = -1) {
   cora_model* m = s->m;
   const cora_model_config& c = m->cfg;
-  const int d = c.d_model, M = s->M;
+  const int d = c.d_model;
+  // cached_block >= 0: a later pass of that block in prefix-cache mode, over
+  // the packed rows lo .. S-1 of every sequence (Ls per sequence).
+  const bool packed = cached_block >= 0;
+  const bool cache = s->opt.cache == CORA_CACHE_PREFIX;
+  const int lo = packed ? s->P + cached_block * s->BL : 0;
+  const int Ls = s->S - lo;
+  const int M = s->B * Ls;
   int* err = s->status + 1;
   cudaStream_t st = s->stream;
   if (rec) {
     rec->st = st;
     rec->mark(-1);
   }
-  launch_embed(s->tokens, m->embed, s->h, M, d, st);
+  launch_embed(s->tokens, m->embed, s->h, M, d, s->S, lo, packed ? Ls : 0, st);
   REC(CORA_KIND_EMBED);
   for (int l = 0; l < c.n_layers; ++l) {
     launch_rmsnorm(s->h, m->attn_norm[l], s->xn, M, d, c.norm_eps, st);
     REC(CORA_KIND_RMSNORM);
-    GemmEpilogue e1{s->qkv, m->n_qkv, CORA_EPI_ROPE_BF16, s->rope, s->S, c.head_dim,
+    uint16_t* qkv = cache ? s->qkv_l[l] : s->qkv;
+    GemmEpilogue e1{qkv, m->n_qkv, CORA_EPI_ROPE_BF16, s->rope, Ls, c.head_dim,
                     (c.n_heads + c.n_kv_heads) * c.head_dim, 1};
-    CK(launch_gemm(s->tm_xn, m->tm_qkv[l], s->tmo_qkv, M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
+    e1.rope_pos0 = lo;
+    e1.out3d = packed ? 1 : 0;
+    const CUtensorMap& tmo = packed ? s->tmo_qkv3_l[l] : cache ? s->tmo_qkv_l[l] : s->tmo_qkv;
+    CK(launch_gemm(s->tm_xn, m->tm_qkv[l], tmo, M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_QKV);
     if (c.head_dim == 128) {
-      CK(launch_attention_tc(s->tm_qkv_in, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, err, st));
+      CK(launch_attention_tc(cache ? s->tm_qkv_in_l[l] : s->tm_qkv_in, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads,
+                             lo, Ls, err, st));
     } else {
-      launch_attention(s->qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, st);
+      launch_attention(qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, lo, Ls, st);
     }
     REC(CORA_KIND_ATTENTION);
     GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0, 1};
@@ -456,8 +475,8 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
     CK(launch_gemm(s->tm_act, m->tm_down[l], s->tmo_h, M, d, m->f_pad, e2, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_DOWN);
   }
-  launch_final_norm_rows(s->h, m->final_norm, s->ctrl, s->xf, s->B, s->S, s->P, s->BL, s->n_blocks, d, c.norm_eps,
-                         s->rows_per_seq, st);
+  launch_final_norm_rows(s->h, m->final_norm, s->ctrl, s->xf, s->B, packed ? Ls : s->S, packed ? -1 : s->P, s->BL,
+                         s->n_blocks, d, c.norm_eps, s->rows_per_seq, st);
   REC(CORA_KIND_FINAL_NORM);
   for (int ch = 0; ch < s->n_chunks; ++ch) {
     const int rows_c = std::min(s->chunk_rows, s->Re - ch * s->chunk_rows);
@@ -468,14 +487,15 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
   SessionGateArgs ga{s->parts, s->n_parts, s->ctrl,  s->tokens, s->state,  s->persist, s->prev,
                      s->conf,  s->argmax,  s->unmask, s->accept, reinterpret_cast<uint8_t*>(s->status),
                      err,      s->B,       s->S,      s->P,      s->G,       s->BL,      s->T,
-                     s->tau,   s->K,       s->opt.schedule, s->opt.eos_id, s->rows_per_seq, s->chunk_rows};
+                     s->tau,   s->K,       s->opt.schedule, s->opt.eos_id, s->rows_per_seq, s->chunk_rows,
+                     cache ? 1 : 0};
   launch_session_gate(ga, st);
   REC(CORA_KIND_GATE);
   CK(cudaGetLastError());
   if (loop)
     CK(launch_step_loop_cond(*loop, s->status, s->max_iters, st));
   else
-    CK(cudaMemcpyAsync(s->status_h, s->status, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+    CK(cudaMemcpyAsync(s->status_h, s->status, (cache ? 4 : 2) * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
   return CORA_OK;
 }
 
@@ -522,6 +542,7 @@ extern "C" int cora_session_reset(cora_session* s, const int32_t* prompt) {
   CK(cudaGetLastError());
   CK(cudaStreamSynchronize(s->stream));
   s->batched_passes = 0;
+  s->next_info = 1;  // the first pass of block 0 is dense
   s->finished = false;
   return CORA_OK;
 }
@@ -537,13 +558,20 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
                                       int32_t gen_len, int32_t block_len, int32_t steps_per_block, float tau,
                                       int32_t K, const cora_decode_options* opt, cora_session** out) {
   REQUIRE(m && out, "cora_session_create: NULL argument");
-  const cora_decode_options o = opt ? *opt : cora_decode_options{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1};
+  const cora_decode_options o = opt ? *opt : cora_decode_options{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1, CORA_CACHE_NONE};
   REQUIRE(o.schedule == CORA_SCHEDULE_FIXED || o.schedule == CORA_SCHEDULE_REMAINING, "unknown schedule %d",
           o.schedule);
   REQUIRE(o.persistence == CORA_PERSIST_BLOCK || o.persistence == CORA_PERSIST_CARRY, "unknown persistence mode %d",
           o.persistence);
   REQUIRE(o.eos_id == -1 || (o.eos_id >= 0 && o.eos_id < m->cfg.vocab && o.eos_id != m->cfg.mask_id),
           "eos_id must be -1 or a vocabulary id other than the mask id");
+  REQUIRE(o.cache == CORA_CACHE_NONE || o.cache == CORA_CACHE_PREFIX, "unknown cache mode %d", o.cache);
+  REQUIRE(o.cache == CORA_CACHE_NONE || o.persistence == CORA_PERSIST_BLOCK,
+          "the prefix cache is not combined with carry-over persistence");
+  // Packed prefix-cache rows are stored in 32-row boxes that must not
+  // straddle two sequences: every suffix length gen_len - b * block_len is
+  // then a multiple of 32.
+  REQUIRE(o.cache == CORA_CACHE_NONE || block_len == 32, "the prefix cache needs block_len == 32");
   REQUIRE(batch >= 1 && prompt_len >= 0 && gen_len >= 1, "bad batch/prompt_len/gen_len");
   REQUIRE(block_len >= 1 && block_len <= 32, "block_len must be in [1, 32]");
   REQUIRE(gen_len % block_len == 0, "gen_len %% block_len != 0");
@@ -585,6 +613,22 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   SK(sess_alloc(s, M * d, &s->h));
   SK(sess_alloc(s, M * d, &s->xn));
   SK(sess_alloc(s, M * size_t(m->n_qkv), &s->qkv));
+  if (o.cache == CORA_CACHE_PREFIX) {
+    for (int l = 0; l < c.n_layers; ++l) {
+      uint16_t* q = nullptr;
+      SK(sess_alloc(s, M * size_t(m->n_qkv), &q));
+      s->qkv_l.push_back(q);
+      CUtensorMap t_out, t_in, t_out3;
+      if (!make_gemm_out_tmap(&t_out, q, int(M), m->n_qkv, CORA_EPI_ROPE_BF16) ||
+          !make_tmap_bf16_2d(&t_in, q, M, size_t(m->n_qkv), size_t(m->n_qkv) * 2, 128, 64) ||
+          !make_tmap_bf16_3d(&t_out3, q, size_t(m->n_qkv), size_t(s->S), size_t(batch), size_t(m->n_qkv) * 2,
+                             size_t(s->S) * m->n_qkv * 2, 64, 32, 1))
+        SK(fail(CORA_ECUDA, "tensor map encoding failed (prefix cache)"));
+      s->tmo_qkv_l.push_back(t_out);
+      s->tm_qkv_in_l.push_back(t_in);
+      s->tmo_qkv3_l.push_back(t_out3);
+    }
+  }
   SK(sess_alloc(s, M * size_t(c.n_heads) * c.head_dim, &s->attn));
   SK(sess_alloc(s, M * size_t(m->f_pad), &s->act));
   SK(sess_alloc(s, size_t(s->Re) * d, &s->xf));
@@ -650,7 +694,28 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
     if (ce != cudaSuccess) SK(fail(CORA_ECUDA, "graph instantiate: %s", cudaGetErrorString(ce)));
   }
   s->max_iters = int32_t(s->n_blocks) * s->T;
-  build_run_graph(s);
+  if (o.cache == CORA_CACHE_PREFIX) {
+    // Later passes of block b: rows P + b * BL .. S-1 of every sequence.
+    for (int b = 0; b < s->n_blocks; ++b) {
+      cudaGraph_t g = nullptr;
+      if (cudaStreamBeginCapture(s->stream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+        SK(fail(CORA_ECUDA, "begin capture"));
+      const int rc = enqueue_step(s, nullptr, nullptr, b);
+      cudaError_t ce = cudaStreamEndCapture(s->stream, &g);
+      if (rc) {
+        if (g) cudaGraphDestroy(g);
+        SK(rc);
+      }
+      if (ce != cudaSuccess) SK(fail(CORA_ECUDA, "end capture: %s", cudaGetErrorString(ce)));
+      cudaGraphExec_t ge = nullptr;
+      ce = cudaGraphInstantiate(&ge, g, 0);
+      cudaGraphDestroy(g);
+      if (ce != cudaSuccess) SK(fail(CORA_ECUDA, "graph instantiate: %s", cudaGetErrorString(ce)));
+      s->cgraph.push_back(ge);
+    }
+  } else {
+    build_run_graph(s);  // (the device loop runs one graph; prefix-cache sessions switch graphs on the host)
+  }
 #undef SK
   *out = s;
   return CORA_OK;
@@ -661,6 +726,7 @@ extern "C" int cora_session_destroy(cora_session* s) {
   if (s->stream) cudaStreamSynchronize(s->stream);
   if (s->graph) cudaGraphExecDestroy(s->graph);
   if (s->run_graph) cudaGraphExecDestroy(s->run_graph);
+  for (auto g : s->cgraph) cudaGraphExecDestroy(g);
   for (void* p : s->allocs) cudaFree(p);
   if (s->status_h) cudaFreeHost(s->status_h);
   if (s->stream) cudaStreamDestroy(s->stream);
@@ -680,8 +746,15 @@ extern "C" int cora_model_destroy(cora_model* m) {
 extern "C" int cora_denoise_step(cora_session* s, uint8_t* all_done_out) {
   REQUIRE(s, "cora_denoise_step: NULL session");
   if (s->finished) return fail(CORA_ESTATE, "every sequence has finished; reset the session");
-  CK(cudaGraphLaunch(s->graph, s->stream));
+  cudaGraphExec_t g = s->graph;
+  if (!s->cgraph.empty() && !(s->next_info & 1)) {
+    const int b = s->next_info >> 1;
+    REQUIRE(b >= 0 && b < int(s->cgraph.size()), "prefix cache: bad block index %d", b);
+    g = s->cgraph[size_t(b)];
+  }
+  CK(cudaGraphLaunch(g, s->stream));
   CK(cudaStreamSynchronize(s->stream));
+  if (!s->cgraph.empty()) s->next_info = s->status_h[3];
   s->batched_passes += 1;
   const int32_t code = s->status_h[1];
   if (code != 0) return fail(CORA_ETIMEOUT, "device error word 0x%x after step", code);
@@ -798,6 +871,11 @@ extern "C" int cora_session_write(cora_session* s, const int32_t* tokens, const 
   if (prev) CK(cudaMemcpy(s->prev, prev, size_t(s->Re) * 4, cudaMemcpyHostToDevice));
   if (ctrl) {
     CK(cudaMemcpy(s->ctrl, ctrl, size_t(s->B) * 16, cudaMemcpyHostToDevice));
+    // Prefix cache: a canvas written at a block's first step (or at another
+    // block) starts with that block's dense pass, which refreshes the kept
+    // keys/values; a later step of the current block keeps them.
+    const int32_t cur = s->next_info >> 1;
+    s->next_info = (ctrl[1] == 0 || ctrl[0] != cur) ? (1 | (ctrl[0] << 1)) : (ctrl[0] << 1);
     bool all = true;
     for (int b = 0; b < s->B; ++b) all = all && ctrl[b * 4 + 3] != 0;
     s->finished = all;
@@ -817,12 +895,12 @@ extern "C" int cora_generate_ex(cora_model* m, const int32_t* prompt, int32_t B,
                                 const cora_decode_options* opt, int32_t* tokens_out, int64_t* passes_out,
                                 int64_t* batched_passes_out) {
   REQUIRE(m && tokens_out && passes_out, "cora_generate: NULL argument");
-  const cora_decode_options o = opt ? *opt : cora_decode_options{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1};
+  const cora_decode_options o = opt ? *opt : cora_decode_options{CORA_SCHEDULE_FIXED, CORA_PERSIST_BLOCK, -1, CORA_CACHE_NONE};
   cora_session* s = m->cached;
   // tau, K and the options are baked into the captured graphs, so they are part of the key.
   if (s && (s->B != B || s->P != P || s->G != gen_len || s->BL != block_len || s->T != steps_per_block ||
             s->tau != tau || s->K != K || s->opt.schedule != o.schedule || s->opt.persistence != o.persistence ||
-            s->opt.eos_id != o.eos_id)) {
+            s->opt.eos_id != o.eos_id || s->opt.cache != o.cache)) {
     cora_session_destroy(s);
     s = nullptr;
   }
@@ -944,9 +1022,9 @@ extern "C" int cora_op_attention(const uint16_t* qkv, uint16_t* out, int32_t B, 
     const size_t cols = size_t(Hq + 2 * Hkv) * hd;
     if (!make_tmap_bf16_2d(&tq, qkv, size_t(B) * S, cols, cols * 2, 128, 64))
       return fail(CORA_ECUDA, "cora_op_attention: tensor map encoding failed");
-    CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, dc->err, static_cast<cudaStream_t>(stream)));
+    CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, 0, S, dc->err, static_cast<cudaStream_t>(stream)));
   } else {
-    launch_attention(qkv, out, B, S, Hq, Hkv, hd, static_cast<cudaStream_t>(stream));
+    launch_attention(qkv, out, B, S, Hq, Hkv, hd, 0, S, static_cast<cudaStream_t>(stream));
   }
   CK(cudaGetLastError());
   return CORA_OK;

@@ -28,14 +28,20 @@ __global__ void synth_normal_bf16_kernel(uint16_t* __restrict__ out, int64_t cou
 }
 
 // h[r, :] = float(embed[tokens[r], :]); one warp per row, 16-byte loads.
+// Row r of h takes token r of the canvas, or, with rows_per_seq > 0 (packed
+// rows of a prefix-cache pass), token lo + r % rows_per_seq of sequence
+// r / rows_per_seq (canvas rows S_tok apart).
 __global__ void embed_kernel(const int32_t* __restrict__ tokens, const uint16_t* __restrict__ embed,
-                             float* __restrict__ h, int M, int d) {
+                             float* __restrict__ h, int M, int d, int S_tok, int lo, int rows_per_seq) {
   pdl_trigger();
   pdl_wait();
   const int row = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   const int lane = threadIdx.x & 31;
   if (row >= M) return;
-  const int tok = tokens[row];
+  const int64_t ti = rows_per_seq > 0
+                         ? static_cast<int64_t>(row / rows_per_seq) * S_tok + lo + row % rows_per_seq
+                         : static_cast<int64_t>(row);
+  const int tok = tokens[ti];
   const uint4* src = reinterpret_cast<const uint4*>(embed + static_cast<int64_t>(tok) * d);
   float4* dst = reinterpret_cast<float4*>(h + static_cast<int64_t>(row) * d);
   for (int c = lane; c < d / 8; c += 32) {
@@ -146,13 +152,15 @@ __global__ void __launch_bounds__(kNormThreads) rmsnorm_kernel(const float* __re
 __global__ void final_norm_rows_kernel(const float* __restrict__ h, const uint16_t* __restrict__ w,
                                        const int32_t* __restrict__ ctrl, uint16_t* __restrict__ out, int B, int S,
                                        int P, int BL, int n_blocks, int d, float eps, int rows_per_seq) {
+  // P < 0: h holds packed prefix-cache rows, S per sequence, with the active
+  // block first.
   pdl_trigger();
   pdl_wait();
   const int r = blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
   if (r >= B * rows_per_seq) return;
   const int b = r / rows_per_seq, i = r % rows_per_seq;
-  int64_t src = static_cast<int64_t>(b) * S + P + i;
-  if (rows_per_seq == BL) {
+  int64_t src = static_cast<int64_t>(b) * S + (P < 0 ? 0 : P) + i;
+  if (rows_per_seq == BL && P >= 0) {
     int blk = ctrl[b * 4 + 0];
     blk = blk < n_blocks ? blk : n_blocks - 1;
     src += static_cast<int64_t>(blk) * BL;
@@ -179,7 +187,7 @@ __global__ void session_init_kernel(int32_t* __restrict__ tokens, const int32_t*
     prev[t] = -1;
   }
   if (t < B * 4) ctrl[t] = 0;
-  if (t < 2) status[t] = 0;
+  if (t < 4) status[t] = t == 3 ? 1 : 0;  // {all_done, error word, loop counter, next pass: dense, block 0}
 }
 
 }  // namespace cora
@@ -206,8 +214,9 @@ void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_
   synth_normal_bf16_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(out, count, key, start, scale);
 }
 
-void launch_embed(const int32_t* tokens, const uint16_t* embed, float* h, int M, int d, cudaStream_t st) {
-  launch_pdl(embed_kernel, dim3((M + 7) / 8), dim3(256), 0, st, tokens, embed, h, M, d);
+void launch_embed(const int32_t* tokens, const uint16_t* embed, float* h, int M, int d, int S_tok, int lo,
+                  int rows_per_seq, cudaStream_t st) {
+  launch_pdl(embed_kernel, dim3((M + 7) / 8), dim3(256), 0, st, tokens, embed, h, M, d, S_tok, lo, rows_per_seq);
 }
 
 void launch_rmsnorm(const float* x, const uint16_t* w, uint16_t* out, int M, int d, float eps, cudaStream_t st) {

@@ -331,3 +331,65 @@ def test_carry_persistence_on_gpu(sharp):
         print(f"carry: {first_pass_accepts} positions accepted on a block's first pass")
     finally:
         cora.cora_session_destroy(s)
+
+
+def replay_compare(m, cfg, w, prompt, options, label):
+    """Replay the oracle's prefix-cache decode step by step: the GPU session is
+    set to the oracle's pre-step state (a block's step 0 makes the pass dense,
+    which keeps the keys/values; later steps reuse them), then Eq. 1 and the
+    gate must agree."""
+    tr = O.generate(cfg, w, prompt[0], G, BL, T, TAU, K, record=True, cache="prefix")
+    s = cora.cora_session_create(m, 1, prompt[:1], P, G, BL, T, TAU, K, options=options)
+    max_dc, cached = 0.0, 0
+    try:
+        for st in tr.steps:
+            b0 = st["before"]
+            ctrl = np.array([[st["block"], st["step"], st["passes_before"], 0]], np.int32)
+            cora.cora_session_write(s, tokens=st["canvas"][None], state=st["gen_state"][None],
+                                    persist=b0.persist[None], prev=b0.prev[None], ctrl=ctrl)
+            cora.cora_denoise_step(s)
+            out = cora.cora_session_read(s, 1, P + G, G, BL)
+            c, a = out["conf"][0], out["argmax"][0]
+            dc = np.abs(c.astype(np.float64) - st["conf"])
+            max_dc = max(max_dc, float(dc.max()))
+            assert dc.max() <= 2e-2, (label, st["block"], st["step"], dc.max())
+            sel = O.top2_margin(st["logits"]) > 2e-2
+            assert np.array_equal(a[sel], st["x_hat"][sel]), (label, st["block"], st["step"])
+            k = O.transfer_schedule(BL, T)[st["step"]]
+            assert rule_holds(b0.state, b0.persist, b0.prev, c, a, k, TAU, K,
+                              dict(unmask=out["unmask"][0], accept=out["accept"][0]))
+            cached += st["step"] > 0
+    finally:
+        cora.cora_session_destroy(s)
+    blocks = {st["block"] for st in tr.steps}
+    print(f"{label}: replayed {len(tr.steps)} steps ({cached} cached passes, blocks {sorted(blocks)}), "
+          f"max|dc| = {max_dc:.2e}")
+    assert cached >= 2 and len(blocks) == G // BL
+
+
+def test_prefix_cache_matches_oracle(tiny):
+    m, w, prompt = tiny
+    replay_compare(m, CFG, w, prompt, cora.decode_options(cache=cora.CACHE_PREFIX), "prefix cache, hd 64")
+
+
+def test_prefix_cache_matches_oracle_hd128():
+    cfg = dict(CFG, name="tiny-hd128", n_heads=2, n_kv_heads=2, head_dim=128)
+    m = model.create_model(cfg, on_device_fill=False)
+    try:
+        w = synth.model_weights_f64(cfg)
+        prompt = synth.prompts(cfg["prompt_seed"], 1, P, cfg["mask_id"])
+        replay_compare(m, cfg, w, prompt, cora.decode_options(cache=cora.CACHE_PREFIX), "prefix cache, hd 128")
+    finally:
+        cora.cora_model_destroy(m)
+
+
+def test_prefix_cache_batch_moves_blocks_together(sharp):
+    """Sequences of a batch move to the next block together; each one's tokens
+    and executed passes are those of a batch of one."""
+    m, prompt = sharp
+    opt = cora.decode_options(cache=cora.CACHE_PREFIX)
+    toks3, passes3, batched = cora.cora_generate(m, prompt, G, BL, T, TAU, K, options=opt)
+    assert batched >= passes3.max()
+    for b in range(prompt.shape[0]):
+        toks1, passes1, _ = cora.cora_generate(m, prompt[b:b + 1], G, BL, T, TAU, K, options=opt)
+        assert passes1[0] == passes3[b] and np.array_equal(toks1[0], toks3[b])
