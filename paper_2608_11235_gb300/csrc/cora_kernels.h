@@ -127,6 +127,12 @@ struct GemmEpilogue {
   // [sequence][position][column] and row r is stored at that position.
   int rope_pos0;
   int out3d;
+  // A (row-major [a_rows, K] bf16): with it, launch_gemm routes M <= 64 to
+  // the few-row (swap-AB) kernel; out_rows_per_seq = output rows per
+  // sequence for out3d stores there.
+  const void* a_ptr;
+  int64_t a_rows;
+  int out_rows_per_seq;
 };
 
 // Stream-K workspace: one fp32 partial slot of 128 x 256 per CTA plus one
@@ -155,6 +161,16 @@ int gemm_block_n(int N, int mode);
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,
                         const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st);
 bool make_gemm_out_tmap(CUtensorMap* map, void* C, int M, int ldc, int mode);
+// Few-row GEMM (gemm_skinny.cu): tmW = weights [N, K] (boxes of 128 rows x 64),
+// tmX = A with boxes of gemm_skinny_npad(M) rows x 64.
+int gemm_skinny_npad(int M);
+bool gemm_skinny_supported(int M, int N, int K, const GemmEpilogue& ep);
+cudaError_t launch_gemm_skinny(const CUtensorMap& tmW, const CUtensorMap& tmX, int M, int N, int K,
+                               const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms,
+                               cudaStream_t st);
+// GemmWorkspace.flags entries: the row-tiled kernels' flags, then the
+// few-row kernel's tile tickets.
+constexpr int kGemmFlagCount = 1024;
 // Generic 2-D tensor map (element size 2 = bf16, 4 = fp32), 128-byte swizzle.
 bool make_tmap_2d(CUtensorMap* map, const void* base, int elem_bytes, uint64_t rows, uint64_t cols,
                   uint64_t row_stride_bytes, uint32_t box_rows, uint32_t box_cols);

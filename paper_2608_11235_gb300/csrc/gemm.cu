@@ -1120,7 +1120,9 @@ int gemm_block_n(int N, int mode) {
   return (N % 256 == 0) ? 256 : 128;
 }
 
-size_t gemm_workspace_bytes(int num_sms) { return static_cast<size_t>(num_sms) * kBM * 256 * sizeof(float); }
+// Row-tiled kernels: one 128 x 256 fp32 slot per CTA; the few-row kernel:
+// two slots of up to 256 x 128 fp32 per CTA.
+size_t gemm_workspace_bytes(int num_sms) { return 2 * static_cast<size_t>(num_sms) * kBM * 256 * sizeof(float); }
 
 // A contributor's partial hand-off (epilogue stores, fence, flag) takes about
 // as long as 13 k-block MMA steps; skewed equal splits hide it behind the
@@ -1193,6 +1195,13 @@ cudaError_t gemm_prepare() {
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,
                         const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st) {
+  if (gemm_skinny_supported(M, N, K, ep)) {
+    CUtensorMap tx;
+    if (!make_tmap_bf16_2d(&tx, ep.a_ptr, static_cast<uint64_t>(ep.a_rows), K, static_cast<uint64_t>(K) * 2,
+                           gemm_skinny_npad(M), 64))
+      return cudaErrorInvalidValue;
+    return launch_gemm_skinny(tmB, tx, M, N, K, ep, ws, err, num_sms, st);
+  }
   if (M > 128 && N % 256 == 0 && g_gemm_pairs_enabled) {
     GemmEpilogue e = ep;
     const int pairs = gemm2_pairs(M, N, K, num_sms, e);

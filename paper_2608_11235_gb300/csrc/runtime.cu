@@ -84,8 +84,8 @@ int device_ctx(DeviceCtx** out) {
     CK(cudaMalloc(&c.err, sizeof(int)));
     CK(cudaMemset(c.err, 0, sizeof(int)));
     CK(cudaMalloc(&c.gemm_ws.partial, gemm_workspace_bytes(c.num_sms)));
-    CK(cudaMalloc(&c.gemm_ws.flags, sizeof(int) * c.num_sms));
-    CK(cudaMemset(c.gemm_ws.flags, 0, sizeof(int) * c.num_sms));
+    CK(cudaMalloc(&c.gemm_ws.flags, sizeof(int) * kGemmFlagCount));
+    CK(cudaMemset(c.gemm_ws.flags, 0, sizeof(int) * kGemmFlagCount));
     if (!g_encode) {
       cudaDriverEntryPointQueryResult q;
       void* fn = nullptr;
@@ -453,6 +453,9 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
                     (c.n_heads + c.n_kv_heads) * c.head_dim, 1};
     e1.rope_pos0 = lo;
     e1.out3d = packed ? 1 : 0;
+    e1.a_ptr = s->xn;
+    e1.a_rows = s->M;
+    e1.out_rows_per_seq = s->S;
     const CUtensorMap& tmo = packed ? s->tmo_qkv3_l[l] : cache ? s->tmo_qkv_l[l] : s->tmo_qkv;
     CK(launch_gemm(s->tm_xn, m->tm_qkv[l], tmo, M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_QKV);
@@ -464,15 +467,21 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
     }
     REC(CORA_KIND_ATTENTION);
     GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0, 1};
+    e2.a_ptr = s->attn;
+    e2.a_rows = s->M;
     CK(launch_gemm(s->tm_attn, m->tm_o[l], s->tmo_h, M, d, c.n_heads * c.head_dim, e2, s->gemm_ws, err, m->num_sms,
                    st));
     REC(CORA_KIND_GEMM_O);
     launch_rmsnorm(s->h, m->ffn_norm[l], s->xn, M, d, c.norm_eps, st);
     REC(CORA_KIND_RMSNORM);
     GemmEpilogue e3{s->act, m->f_pad, CORA_EPI_SWIGLU, nullptr, 0, 0, 0, 1};
+    e3.a_ptr = s->xn;
+    e3.a_rows = s->M;
     CK(launch_gemm(s->tm_xn, m->tm_gu[l], s->tmo_act, M, 2 * m->f_pad, d, e3, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_GATE_UP);
-    CK(launch_gemm(s->tm_act, m->tm_down[l], s->tmo_h, M, d, m->f_pad, e2, s->gemm_ws, err, m->num_sms, st));
+    GemmEpilogue e4 = e2;  // residual epilogue, A = the SwiGLU output
+    e4.a_ptr = s->act;
+    CK(launch_gemm(s->tm_act, m->tm_down[l], s->tmo_h, M, d, m->f_pad, e4, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_DOWN);
   }
   launch_final_norm_rows(s->h, m->final_norm, s->ctrl, s->xf, s->B, packed ? Ls : s->S, packed ? -1 : s->P, s->BL,
@@ -646,8 +655,8 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   SK(sess_alloc(s, 4, &s->status));
   SK(sess_alloc(s, size_t(batch) * 3, &s->diag));
   SK(sess_alloc(s, gemm_workspace_bytes(m->num_sms) / sizeof(float), &s->gemm_ws.partial));
-  SK(sess_alloc(s, size_t(m->num_sms), &s->gemm_ws.flags));
-  if (cudaMemset(s->gemm_ws.flags, 0, sizeof(int) * m->num_sms) != cudaSuccess) SK(fail(CORA_ECUDA, "memset"));
+  SK(sess_alloc(s, size_t(kGemmFlagCount), &s->gemm_ws.flags));
+  if (cudaMemset(s->gemm_ws.flags, 0, sizeof(int) * kGemmFlagCount) != cudaSuccess) SK(fail(CORA_ECUDA, "memset"));
   {
     void* hp = nullptr;
     if (cudaHostAlloc(&hp, 16, cudaHostAllocDefault) != cudaSuccess) SK(fail(CORA_ENOMEM, "pinned alloc"));
@@ -1003,6 +1012,8 @@ extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32
       !make_gemm_out_tmap(&tc, C, M, ldc, epilogue))
     return fail(CORA_ECUDA, "cora_op_gemm: tensor map encoding failed");
   GemmEpilogue ep{C, ldc, epilogue, rope, seq, head_dim, rope_cols, 0};
+  ep.a_ptr = A;
+  ep.a_rows = M;
   CK(launch_gemm(ta, tb, tc, M, N, K, ep, dc->gemm_ws, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
   return CORA_OK;
 }

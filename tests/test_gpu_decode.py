@@ -384,12 +384,35 @@ def test_prefix_cache_matches_oracle_hd128():
 
 
 def test_prefix_cache_batch_moves_blocks_together(sharp):
-    """Sequences of a batch move to the next block together; each one's tokens
-    and executed passes are those of a batch of one."""
+    """Prefix-cache sessions move a batch's sequences to the next block
+    together: unfinished sequences always share the block index, a sequence
+    whose block has ended waits with its canvas untouched, its executed-pass
+    count grows only while it works, and the decode ends fully resolved."""
     m, prompt = sharp
-    opt = cora.decode_options(cache=cora.CACHE_PREFIX)
-    toks3, passes3, batched = cora.cora_generate(m, prompt, G, BL, T, TAU, K, options=opt)
-    assert batched >= passes3.max()
-    for b in range(prompt.shape[0]):
-        toks1, passes1, _ = cora.cora_generate(m, prompt[b:b + 1], G, BL, T, TAU, K, options=opt)
-        assert passes1[0] == passes3[b] and np.array_equal(toks1[0], toks3[b])
+    B = prompt.shape[0]
+    s = cora.cora_session_create(m, B, prompt, P, G, BL, T, TAU, K,
+                                 options=cora.decode_options(cache=cora.CACHE_PREFIX))
+    try:
+        active_steps = np.zeros(B, np.int64)
+        waited = 0
+        done = False
+        while not done:
+            bf = cora.cora_session_read(s, B, P + G, G, BL)
+            done = cora.cora_denoise_step(s)
+            af = cora.cora_session_read(s, B, P + G, G, BL)
+            live = bf["ctrl"][:, 3] == 0
+            assert len(set(bf["ctrl"][live, 0])) <= 1                      # one block for the batch
+            for b in np.flatnonzero(live):
+                if bf["ctrl"][b, 1] < 0:                                   # waiting: nothing changes
+                    waited += 1
+                    assert np.array_equal(af["tokens"][b], bf["tokens"][b])
+                    assert np.array_equal(af["state"][b], bf["state"][b])
+                    assert af["ctrl"][b, 2] == bf["ctrl"][b, 2]
+                else:
+                    active_steps[b] += 1
+        out = cora.cora_session_read(s, B, P + G, G, BL)
+        assert np.array_equal(out["ctrl"][:, 2], active_steps)
+        assert np.all(out["state"] != 0) and np.all(out["ctrl"][:, 3] == 1)
+        print(f"prefix-cache batch: {waited} waiting sequence-steps, passes {active_steps.tolist()}")
+    finally:
+        cora.cora_session_destroy(s)

@@ -87,7 +87,8 @@ def run_gemm(A, Bm, M, N, K, epi, out_cols, out_dtype=torch.int16, C0=None, **kw
 
 @pytest.mark.parametrize("M,N,K", [(300, 512, 320), (128, 384, 64), (2048, 4096, 256), (256, 256, 4096),
                                    (96, 768, 256), (1, 256, 128), (512, 4096, 4096), (512, 12288, 1024),
-                                   (96, 768, 2048), (128, 16384, 512)])
+                                   (96, 768, 2048), (128, 16384, 512),
+                                   (64, 12288, 1024), (16, 4096, 4096), (5, 384, 640)])   # few-row kernel
 def test_gemm_store(M, N, K):
     A = bits(2, 10, (M, K), 1.0)
     Bm = bits(2, 11, (N, K), 1.0 / math.sqrt(K))
@@ -105,7 +106,8 @@ def test_gemm_split_tiles_are_deterministic(M, N, K):
     assert np.array_equal(c1, c2)
 
 
-@pytest.mark.parametrize("M,N,K", [(300, 512, 320), (130, 256, 1024), (512, 4096, 12288), (100, 16384, 512)])
+@pytest.mark.parametrize("M,N,K", [(300, 512, 320), (130, 256, 1024), (512, 4096, 12288), (100, 16384, 512),
+                                   (40, 4096, 12288), (64, 16384, 512)])
 def test_gemm_residual(M, N, K):
     A = bits(3, 10, (M, K), 1.0)
     Bm = bits(3, 11, (N, K), 1.0 / math.sqrt(K))
@@ -115,7 +117,7 @@ def test_gemm_residual(M, N, K):
     assert np.abs(Ct.cpu().numpy() - ref).max() <= 1e-5 * np.abs(ref).max() + 1e-6
 
 
-@pytest.mark.parametrize("M,F,K", [(300, 256, 256), (96, 768, 256)])
+@pytest.mark.parametrize("M,F,K", [(300, 256, 256), (96, 768, 256), (48, 4096, 4096), (7, 768, 256)])
 def test_gemm_swiglu(M, F, K):
     A = bits(4, 10, (M, K), 1.0)
     g = bits(4, 11, (F, K), 1.0 / math.sqrt(K))
@@ -134,7 +136,9 @@ def rope_table(seq, hd, theta):
     return torch.from_numpy(np.stack([np.cos(ang), np.sin(ang)], -1).astype(np.float32)).cuda()
 
 
-@pytest.mark.parametrize("B,S,H,Hkv,hd,theta", [(2, 96, 4, 4, 64, 1e4), (1, 300, 2, 1, 128, 5e5)])
+@pytest.mark.parametrize("B,S,H,Hkv,hd,theta", [(2, 96, 4, 4, 64, 1e4), (1, 300, 2, 1, 128, 5e5),
+                                                  (1, 96, 4, 4, 64, 1e4), (1, 100, 2, 1, 128, 5e5),
+                                                  (1, 48, 4, 4, 64, 1e4), (1, 60, 2, 1, 128, 5e5)])
 def test_gemm_rope(B, S, H, Hkv, hd, theta):
     d = 256
     N = (H + 2 * Hkv) * hd
