@@ -361,7 +361,10 @@ CORA_API int cora_reduce_gate(const uint16_t* logits, int32_t B, int32_t R, int3
  *   C     bf16 [M, ldc] (STORE, ROPE, SWIGLU) or fp32 [M, ldc] (RESID)
  *   rope  fp32 [seq, head_dim/2, 2] (cos, sin) table for ROPE, else NULL
  * Constraints: K % 64 == 0, N % 128 == 0 (SWIGLU: N % 256 == 0), M >= 1,
- * pointers 16-byte aligned, row strides multiples of 16 bytes. */
+ * pointers 16-byte aligned, row strides multiples of 16 bytes.
+ * With ROPE the call also enqueues a transposed copy of the table into
+ * stream-ordered memory (cudaMallocAsync on `stream`, freed after the GEMM):
+ * the tile epilogue reads it frequency-major. */
 CORA_API int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32_t M, int32_t N, int32_t K, int32_t ldc,
                  int32_t epilogue, const float* rope, int32_t seq, int32_t head_dim, int32_t rope_cols,
                  void* stream);

@@ -105,11 +105,13 @@ void launch_gate_transfer(const GateBuffers& gb, int B, int R, int k, float tau,
 void launch_session_gate(const SessionGateArgs& a, cudaStream_t st);
 
 // GEMM (tcgen05).  Epilogue parameters.
+// rope [seq][half][2] -> rope_t [half][seq][2].
+void launch_rope_transpose(const float* rope, float* rope_t, int seq, int half, cudaStream_t st);
 struct GemmEpilogue {
   void* C;
   int ldc;
   int mode;             // CORA_EPI_*
-  const float* rope;    // [seq][head_dim/2][2]
+  const float* rope;    // [seq][head_dim/2][2] (position-major; the few-row kernel)
   int seq;
   int head_dim;
   int rope_cols;
@@ -133,6 +135,12 @@ struct GemmEpilogue {
   const void* a_ptr;
   int64_t a_rows;
   int out_rows_per_seq;
+  // The same RoPE table frequency-major, [head_dim/2][rope_tn][2]: the
+  // row-tiled kernels' epilogue thread owns one row (position), so a warp
+  // reads one frequency for 32 consecutive positions in one 256-byte line
+  // pair instead of 32 lines.
+  const float* rope_t;
+  int rope_tn;
 };
 
 // Stream-K workspace: one fp32 partial slot of 128 x 256 per CTA plus one

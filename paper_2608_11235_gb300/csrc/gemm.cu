@@ -28,6 +28,8 @@
 // segment overlap the MMAs of the next.
 #include <math.h>
 
+#include <algorithm>
+
 #include "cora_device.cuh"
 #include "cora_kernels.h"
 #include "../../include/cora.h"
@@ -140,7 +142,10 @@ __device__ __forceinline__ void red_add_v4(float* dst, const float* a) {
                : "memory");
 }
 
-__device__ __forceinline__ float silu_f(float x) { return x / (1.f + __expf(-x)); }
+// silu(x) = x / (1 + e^-x); the approximate divide is within 2 ulp (the
+// result is rounded to bf16), and for x -> -inf the denominator overflows to
+// inf and the quotient goes to -0 as the exact function does.
+__device__ __forceinline__ float silu_f(float x) { return __fdividef(x, 1.f + __expf(-x)); }
 
 __device__ __forceinline__ void store_bf16x16(uint16_t* dst, const float (&v)[16]) {
   uint4 a, b;
@@ -370,7 +375,7 @@ __device__ __forceinline__ void gemm_epilogue_warp(const GemmEpilogue& ep, const
     const int pos = ep.rope_pos0 + (row0 + lane >= 0 ? (row0 + lane) % ep.seq : 0);
     // store coordinates of the warp's 32-row box (they never straddle a sequence: seq % 32 == 0 when out3d)
     const int srow = ep.out3d ? ep.rope_pos0 + row0 % ep.seq : row0, sseq = ep.out3d ? row0 / ep.seq : -1;
-    const float2* tab = reinterpret_cast<const float2*>(ep.rope) + static_cast<int64_t>(pos) * half;
+    const float2* tab = reinterpret_cast<const float2*>(ep.rope_t) + pos;  // frequency j at tab[j * rope_tn]
 #pragma unroll 1
     for (int h0 = 0; h0 < BN; h0 += hd) {
       const bool rot = n0 + h0 < ep.rope_cols;
@@ -397,7 +402,7 @@ __device__ __forceinline__ void gemm_epilogue_warp(const GemmEpilogue& ep, const
           for (int q = 0; q < 2; ++q)
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
-              const float2 cs = tab[j0 + 16 * q + j];
+              const float2 cs = tab[static_cast<int64_t>(j0 + 16 * q + j) * ep.rope_tn];
               const float a = v[q][j], b = v[q + 2][j];
               v[q][j] = a * cs.x - b * cs.y;
               v[q + 2][j] = b * cs.x + a * cs.y;
@@ -1211,6 +1216,22 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
   if (gemm_block_n(N, ep.mode) == 256)
     return launch_gemm_bn<256>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);
   return launch_gemm_bn<128>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);
+}
+
+__global__ void rope_transpose_kernel(const float2* __restrict__ rope, float2* __restrict__ rope_t, int seq, int half) {
+  const int64_t n = static_cast<int64_t>(seq) * half;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t j = i / seq, p = i - j * seq;  // output index i = j * seq + p
+    rope_t[i] = rope[p * half + j];
+  }
+}
+
+void launch_rope_transpose(const float* rope, float* rope_t, int seq, int half, cudaStream_t st) {
+  const int64_t n = static_cast<int64_t>(seq) * half;
+  const int blocks = static_cast<int>(std::min<int64_t>((n + 255) / 256, 1024));
+  rope_transpose_kernel<<<blocks, 256, 0, st>>>(reinterpret_cast<const float2*>(rope), reinterpret_cast<float2*>(rope_t),
+                                                seq, half);
 }
 
 // Output tensor map of a GEMM: 32-row x 128-byte boxes, 128-byte swizzle

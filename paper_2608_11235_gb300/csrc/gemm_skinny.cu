@@ -59,7 +59,8 @@ struct SkCfg {
 // its 32 consecutive rows covers 512 contiguous bytes.
 __device__ __forceinline__ int64_t sk_f4(int m, int n, int tr) { return static_cast<int64_t>(m >> 2) * tr + n; }
 
-__device__ __forceinline__ float silu_sk(float x) { return x / (1.f + __expf(-x)); }
+// silu as in the row-tiled kernels (approximate divide, bf16 result)
+__device__ __forceinline__ float silu_sk(float x) { return __fdividef(x, 1.f + __expf(-x)); }
 
 template <int NPAD, int TR>
 __global__ void __launch_bounds__(192, 1)
@@ -272,11 +273,19 @@ __global__ void __launch_bounds__(192, 1)
             }
         }
         if (ep.mode == CORA_EPI_RESID_F32) {
+          // all 16 residuals loaded before any store: one memory round trip
+          // per chunk instead of a chain of 16 read-add-writes
           float* C = static_cast<float*>(ep.C);
+          float res[16];
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             const int m = m0 + j;
-            if (m < M) C[static_cast<int64_t>(m) * ep.ldc + n_glob] += v[0][j];
+            res[j] = m < M ? __ldcg(C + static_cast<int64_t>(m) * ep.ldc + n_glob) : 0.f;
+          }
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int m = m0 + j;
+            if (m < M) C[static_cast<int64_t>(m) * ep.ldc + n_glob] = res[j] + v[0][j];
           }
         } else if (ep.mode == CORA_EPI_SWIGLU) {
           uint16_t* C = static_cast<uint16_t*>(ep.C);
@@ -298,18 +307,22 @@ __global__ void __launch_bounds__(192, 1)
             named_bar_sync(1, 128);
             const int pn = nl ^ half;
             const int jj = static_cast<int>(n_glob % hd);
-            float r[16];
+            // the chunk's 16 (cos, sin) pairs loaded together, ahead of their use
+            float2 cs[16];
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
               const int m = m0 + j;
+              cs[j] = rope && m < M ? __ldg(reinterpret_cast<const float2*>(ep.rope) +
+                                            static_cast<int64_t>(ep.rope_pos0 + m % ep.seq) * half + (jj % half))
+                                    : make_float2(1.f, 0.f);
+            }
+            float r[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) {
               const float other = ex[pn * 16 + ((j + (pn & 31)) & 15)];
-              if (rope && m < M) {
-                const int pos = ep.rope_pos0 + m % ep.seq;
-                const float2 cs = reinterpret_cast<const float2*>(ep.rope)[static_cast<int64_t>(pos) * half + (jj % half)];
-                r[j] = jj < half ? v[0][j] * cs.x - other * cs.y : v[0][j] * cs.x + other * cs.y;
-              } else {
-                r[j] = v[0][j];
-              }
+              r[j] = !rope ? v[0][j]
+                     : jj < half ? v[0][j] * cs[j].x - other * cs[j].y
+                                 : v[0][j] * cs[j].x + other * cs[j].y;
             }
             named_bar_sync(1, 128);  // ex is rewritten by the next chunk
 #pragma unroll

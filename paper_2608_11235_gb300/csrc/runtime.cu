@@ -343,6 +343,7 @@ struct cora_session {
   uint16_t* act = nullptr;     // [M, f_pad]
   uint16_t* xf = nullptr;      // [R, d] final-normed active rows
   float* rope = nullptr;       // [S, hd/2, 2]
+  float* rope_t = nullptr;     // [hd/2, S, 2] (the same table, frequency-major)
   Top1Part* parts = nullptr;   // [n_parts, R]
   int n_parts = 0;
   int32_t* ctrl = nullptr;     // [B, 4]
@@ -452,6 +453,8 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
     GemmEpilogue e1{qkv, m->n_qkv, CORA_EPI_ROPE_BF16, s->rope, Ls, c.head_dim,
                     (c.n_heads + c.n_kv_heads) * c.head_dim, 1};
     e1.rope_pos0 = lo;
+    e1.rope_t = s->rope_t;
+    e1.rope_tn = s->S;
     e1.out3d = packed ? 1 : 0;
     e1.a_ptr = s->xn;
     e1.a_rows = s->M;
@@ -642,6 +645,7 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   SK(sess_alloc(s, M * size_t(m->f_pad), &s->act));
   SK(sess_alloc(s, size_t(s->Re) * d, &s->xf));
   SK(sess_alloc(s, size_t(s->S) * c.head_dim, &s->rope));
+  SK(sess_alloc(s, size_t(s->S) * c.head_dim, &s->rope_t));
   s->n_parts = lm_head_parts_count(c.vocab, m->num_sms);
   SK(sess_alloc(s, size_t(s->n_parts) * s->n_chunks * s->chunk_rows, &s->parts));
   SK(sess_alloc(s, size_t(batch) * 4, &s->ctrl));
@@ -672,7 +676,12 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
         tab[(size_t(p) * half + j) * 2] = float(std::cos(ang));
         tab[(size_t(p) * half + j) * 2 + 1] = float(std::sin(ang));
       }
-    if (cudaMemcpy(s->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
+    std::vector<float> tab_t(tab.size());
+    for (int p = 0; p < s->S; ++p)
+      for (int j = 0; j < half; ++j)
+        for (int e = 0; e < 2; ++e) tab_t[(size_t(j) * s->S + p) * 2 + e] = tab[(size_t(p) * half + j) * 2 + e];
+    if (cudaMemcpy(s->rope, tab.data(), tab.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemcpy(s->rope_t, tab_t.data(), tab_t.size() * 4, cudaMemcpyHostToDevice) != cudaSuccess)
       SK(fail(CORA_ECUDA, "rope table upload"));
   }
   const size_t hq = size_t(c.n_heads) * c.head_dim;
@@ -1014,7 +1023,19 @@ extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32
   GemmEpilogue ep{C, ldc, epilogue, rope, seq, head_dim, rope_cols, 0};
   ep.a_ptr = A;
   ep.a_rows = M;
-  CK(launch_gemm(ta, tb, tc, M, N, K, ep, dc->gemm_ws, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* rope_t = nullptr;
+  if (epilogue == CORA_EPI_ROPE_BF16) {
+    // the row-tiled epilogue reads the table frequency-major: a stream-ordered
+    // transposed copy, released after the GEMM
+    CK(cudaMallocAsync(reinterpret_cast<void**>(&rope_t), size_t(seq) * head_dim * sizeof(float), st));
+    launch_rope_transpose(rope, rope_t, seq, head_dim / 2, st);
+    ep.rope_t = rope_t;
+    ep.rope_tn = seq;
+  }
+  const cudaError_t ge = launch_gemm(ta, tb, tc, M, N, K, ep, dc->gemm_ws, dc->err, dc->num_sms, st);
+  if (rope_t) CK(cudaFreeAsync(rope_t, st));
+  CK(ge);
   return CORA_OK;
 }
 
