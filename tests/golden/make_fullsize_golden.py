@@ -11,6 +11,13 @@ generator are called.
 
 Output: tests/golden/fullsize_<preset>.json (conf, argmax, top-1/top-2
 probability margin and logit gap per row, for each head).
+
+    python tests/golden/make_fullsize_golden.py --blocks [preset ...]
+
+Later blocks: the same pass on seeded mid-decode canvases
+(synth.mid_decode_canvas): the first pass of blocks 1, 4 and 7 and two
+passes inside blocks 3 and 6 with part of the block already resolved.
+Output: tests/golden/fullsize_<preset>_blocks.json.
 """
 
 from __future__ import annotations
@@ -45,6 +52,38 @@ def head_eq1(cfg, rows, v_chunk=16384):
             "logit_gap": (srt[:, -1] - srt[:, -2]).tolist()}
 
 
+CANVAS_SEED = 500
+BLOCK_CASES = [(1, 0.0), (4, 0.0), (7, 0.0), (3, 0.5), (6, 0.75)]  # (active block, fraction already resolved)
+
+
+def forward_rows(cfg, tokens, block, tag):
+    """Oracle hidden states of the active block's rows after the last layer."""
+    P, BL = cfg["prompt_len"], cfg["block_len"]
+    h = np.stack([synth.weight_f64(cfg, -1, synth.EMBED, slice(int(t), int(t) + 1))[0] for t in tokens])
+    pos = np.arange(len(tokens))
+    t0 = time.time()
+    for l in range(cfg["n_layers"]):
+        h = O.layer_forward(cfg, synth.layer_weights_f64(cfg, l), h, pos)
+        print(f"{tag}: layer {l} done at {time.time() - t0:.0f} s", flush=True)
+    return h[P + block * BL: P + (block + 1) * BL]
+
+
+def run_blocks(preset: str) -> None:
+    cfg = dict(configs.PRESETS[preset])
+    cases = []
+    for block, frac in BLOCK_CASES:
+        tokens, state = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, frac)
+        rows = forward_rows(cfg, tokens, block, f"{preset} block {block} frac {frac}")
+        cases.append({"block": block, "frac_resolved": frac, "canvas_seed": CANVAS_SEED,
+                      "heads": {"workload": head_eq1(cfg, rows),
+                                "gate_exercising": head_eq1(configs.gate_exercising(cfg), rows)}})
+    out = {"preset": preset, "sequence": 0,
+           "source": "oracle/cora_oracle.py (layer_forward, lm_logits, top1, top2_margin), float64",
+           "cases": cases}
+    with open(os.path.join(HERE, f"fullsize_{preset}_blocks.json"), "w") as f:
+        json.dump(out, f)
+
+
 def run(preset: str) -> None:
     cfg = dict(configs.PRESETS[preset])
     P, G, BL = cfg["prompt_len"], cfg["gen_len"], cfg["block_len"]
@@ -66,5 +105,10 @@ def run(preset: str) -> None:
 
 
 if __name__ == "__main__":
-    for p in (sys.argv[1:] or PRESETS):
-        run(p)
+    args = sys.argv[1:]
+    if args and args[0] == "--blocks":
+        for p in (args[1:] or PRESETS[:1]):
+            run_blocks(p)
+    else:
+        for p in (args or PRESETS):
+            run(p)
