@@ -14,9 +14,9 @@ probability margin and logit gap per row, for each head).
 
     python tests/golden/make_fullsize_golden.py --blocks [preset ...]
 
-Later blocks: the same pass on seeded mid-decode canvases
-(synth.mid_decode_canvas): the first pass of blocks 1, 4 and 7 and two
-passes inside blocks 3 and 6 with part of the block already resolved.
+Later blocks: the same pass on seeded mid-decode canvases of sequence 0
+(synth.mid_decode_canvas), per workload in BLOCK_CASES: first passes of
+later blocks and passes inside a block with part of it already resolved.
 Output: tests/golden/fullsize_<preset>_blocks.json.
 """
 
@@ -53,7 +53,12 @@ def head_eq1(cfg, rows, v_chunk=16384):
 
 
 CANVAS_SEED = 500
-BLOCK_CASES = [(1, 0.0), (4, 0.0), (7, 0.0), (3, 0.5), (6, 0.75)]  # (active block, fraction already resolved)
+# (active block, fraction of it already resolved) per workload
+BLOCK_CASES = {
+    "llada8b-shape-256+256": [(1, 0.0), (4, 0.0), (7, 0.0), (3, 0.5), (6, 0.75)],
+    "dream7b-shape-256+512-b4": [(5, 0.0), (15, 0.0), (10, 0.5)],
+    "llada8b-shape-512+1024-b8": [(15, 0.0), (31, 0.0)],
+}
 
 
 def forward_rows(cfg, tokens, block, tag):
@@ -71,7 +76,7 @@ def forward_rows(cfg, tokens, block, tag):
 def run_blocks(preset: str) -> None:
     cfg = dict(configs.PRESETS[preset])
     cases = []
-    for block, frac in BLOCK_CASES:
+    for block, frac in BLOCK_CASES[preset]:
         tokens, state = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, frac)
         rows = forward_rows(cfg, tokens, block, f"{preset} block {block} frac {frac}")
         cases.append({"block": block, "frac_resolved": frac, "canvas_seed": CANVAS_SEED,

@@ -134,3 +134,71 @@ def test_later_blocks_parity_full_size():
         finally:
             cora.cora_model_destroy(m)
             torch.cuda.empty_cache()
+
+
+# Steps checked per workload: every executed step of the whole decode for the
+# 256 + 256 and Dream-shaped workloads; the first four blocks of every
+# sequence for the 512 + 1024 x 8 workload (~14 passes per block at ~0.1 s).
+GATE_BLOCKS = {"llada8b-shape-256+256": None, "dream7b-shape-256+512-b4": None, "llada8b-shape-512+1024-b8": 4}
+
+
+@pytest.mark.parametrize("preset", PRESETS)
+def test_gate_every_step_full_size(preset):
+    """Eq. 2-4 and block termination, bit-exact at every executed step of the
+    full-size decode: before each cora_denoise_step the session's state is
+    read; the oracle's step (oracle.cora_step) is applied to that state with
+    the GPU's own Eq. 1 outputs (float32 confidence, argmax) of the step; its
+    transfer and acceptance sets, canvas, position states, persistence and
+    control must equal the GPU's.  Gate-exercising head, so the gate fires."""
+    from oracle import cora_oracle as O
+    cfg = configs.gate_exercising(configs.PRESETS[preset])
+    B, P, G, BL, T = cfg["batch"], cfg["prompt_len"], cfg["gen_len"], cfg["block_len"], cfg["steps_per_block"]
+    tau, K = cfg["tau"], cfg["K"]
+    n_blocks = G // BL
+    stop_block = GATE_BLOCKS[preset] or n_blocks
+    ks = O.transfer_schedule(BL, T)
+    prompts = synth.prompts(cfg["prompt_seed"], B, P, cfg["mask_id"])
+    m = model.create_model(cfg)
+    steps = accepted = blocks_done = 0
+    try:
+        s = cora.cora_session_create(m, B, prompts, P, G, BL, T, tau, K)
+        try:
+            before = cora.cora_session_read(s, B, P + G, G, BL)
+            while np.any(before["ctrl"][:, 0] < stop_block):
+                cora.cora_denoise_step(s)
+                after = cora.cora_session_read(s, B, P + G, G, BL)
+                for b in range(B):
+                    blk, step = int(before["ctrl"][b, 0]), int(before["ctrl"][b, 1])
+                    if blk >= n_blocks:
+                        assert np.array_equal(after["ctrl"][b], before["ctrl"][b])  # finished: untouched
+                        continue
+                    g0, p0 = blk * BL, P + blk * BL
+                    st = O.BlockState(before["tokens"][b, p0:p0 + BL].astype(np.int64),
+                                      before["state"][b, g0:g0 + BL].copy(),
+                                      before["persist"][b].astype(np.int64), before["prev"][b].astype(np.int64))
+                    r = O.cora_step(st, after["conf"][b], after["argmax"][b].astype(np.int64), ks[step], tau, K)
+                    lbl = (preset, b, blk, step)
+                    assert sorted(np.flatnonzero(after["unmask"][b])) == r.transferred, lbl
+                    assert sorted(np.flatnonzero(after["accept"][b])) == r.accepted, lbl
+                    assert np.array_equal(after["tokens"][b, p0:p0 + BL], st.tokens), lbl
+                    assert np.array_equal(after["state"][b, g0:g0 + BL], st.state), lbl
+                    assert np.array_equal(after["tokens"][b, :p0], before["tokens"][b, :p0]), lbl
+                    assert after["ctrl"][b, 2] == before["ctrl"][b, 2] + 1, lbl
+                    if r.done:
+                        assert after["ctrl"][b, 0] == blk + 1 and after["ctrl"][b, 1] == 0, lbl
+                        blocks_done += 1
+                    else:
+                        assert after["ctrl"][b, 0] == blk and after["ctrl"][b, 1] == step + 1, lbl
+                        assert np.array_equal(after["persist"][b], st.persist), lbl
+                        assert np.array_equal(after["prev"][b], st.prev), lbl
+                    steps += 1
+                    accepted += len(r.accepted)
+                before = after
+        finally:
+            cora.cora_session_destroy(s)
+        assert cora.cora_device_error() == 0
+    finally:
+        cora.cora_model_destroy(m)
+        torch.cuda.empty_cache()
+    assert accepted > 0 and blocks_done >= B
+    print(f"{preset}: {steps} sequence-steps checked, {blocks_done} blocks ended, {accepted} positions accepted")
