@@ -64,7 +64,7 @@ def test_device_generator_bit_exact(seed, stream, sigma, start):
 
 
 # ----------------------------------------------------------------- RMSNorm
-@pytest.mark.parametrize("M,d", [(1, 256), (97, 4096), (33, 3584), (5, 8192)])
+@pytest.mark.parametrize("M,d", [(1, 256), (97, 4096), (33, 3584), (5, 8192), (512, 4096), (607, 3584), (1000, 4096)])
 def test_rmsnorm(M, d):
     x = f64(bits(1, 1, (M, d), 0.7)).astype(np.float32)
     w = bits(1, 2, (d,), 1.0)
