@@ -46,8 +46,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # by a hash of the kernel source at capture time; null once the source changed.
 NCU_TRAFFIC = {
     # gemm_tc2_kernel, mean of the QKV / O / gate-up / down launches (read + write):
-    # (125.4 + 46.4 + 245.3 + 125.8) MB / 4, profiles/gemm_tc2_llada8b_256.md
-    ("gemm", "669151893cf6"): 135_732_000,
+    # (126.0 + 46.3 + 246.3 + 125.5) MB / 4, profiles/gemm_tc2_llada8b_256.md
+    ("gemm", "2f06f7bcf379"): 136_028_000,
 }
 
 
