@@ -18,6 +18,8 @@
 // softmax warps never wait for a PV in the common case.
 // Two TMEM buffers for S and two P buffers let the softmax of tile j overlap
 // the MMAs of tiles j-1 and j+1.  TMEM: S[0] +0, S[1] +128, O +256.
+// K and V buffers are released separately (K_j once QK_j is done, V_j once
+// PV_j is), so K_{j+2} streams in while tile j is still in the softmax.
 // Warps: 0 = TMA producer, 1 = TMEM allocator + MMA issuer, 2..5 = softmax and
 // output.  Keys beyond the sequence end are masked; the output is written by
 // TMA through a [sequence][row][column] map, which clips rows beyond the end.
@@ -112,13 +114,15 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t* sP[2] = {smem + 5 * OPND, smem + 6 * OPND};
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 7 * OPND);
   uint64_t* qfull = bars + 0;
-  uint64_t* kvfull = bars + 1;   // [2] K_j, V_j landed
-  uint64_t* kvempty = bars + 3;  // [2] QK_j and PV_j done with K_j, V_j
-  uint64_t* sfull = bars + 5;    // [2] S_j in TMEM
-  uint64_t* sfree = bars + 7;    // [2] S_j read out by the four softmax warps
-  uint64_t* pfull = bars + 9;    // [2] P_j written (and O rescaled, if it was)
-  uint64_t* pdone = bars + 11;   // [2] PV_j complete (P buffer free, O up to date)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 13);
+  uint64_t* kfull = bars + 1;    // [2] K_j landed
+  uint64_t* vfull = bars + 3;    // [2] V_j landed
+  uint64_t* kempty = bars + 5;   // [2] QK_j done with K_j
+  uint64_t* vempty = bars + 7;   // [2] PV_j done with V_j
+  uint64_t* sfull = bars + 9;    // [2] S_j in TMEM
+  uint64_t* sfree = bars + 11;   // [2] S_j read out by the four softmax warps
+  uint64_t* pfull = bars + 13;   // [2] P_j written (and O rescaled, if it was)
+  uint64_t* pdone = bars + 15;   // [2] PV_j complete (P buffer free, O up to date)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -132,8 +136,10 @@ __global__ void __launch_bounds__(192, 1)
   if (threadIdx.x == 0) {
     mbar_init(qfull, 1);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&kvfull[i], 1);
-      mbar_init(&kvempty[i], 1);
+      mbar_init(&kfull[i], 1);
+      mbar_init(&vfull[i], 1);
+      mbar_init(&kempty[i], 1);
+      mbar_init(&vempty[i], 1);
       mbar_init(&sfull[i], 1);
       mbar_init(&sfree[i], 4);
       mbar_init(&pfull[i], 4);
@@ -165,13 +171,16 @@ __global__ void __launch_bounds__(192, 1)
       tma_load_2d(sQ + OPND / 2, &tmQKV, qfull, qcol + 64, row_base + q0);
       for (int j = 0; j < n_kt; ++j) {
         const int s = j & 1;
-        if (!mbar_wait(&kvempty[s], ((j >> 1) & 1) ^ 1u, abort_flag, err, CORA_DERR_TMA_WAIT)) break;
-        mbar_arrive_expect_tx(&kvfull[s], 2 * OPND);
+        const uint32_t ph = ((j >> 1) & 1) ^ 1u;
         const int r = row_base + j * KT;
-        tma_load_2d(sK[s], &tmQKV, &kvfull[s], kcol, r);
-        tma_load_2d(sK[s] + OPND / 2, &tmQKV, &kvfull[s], kcol + 64, r);
-        tma_load_2d(sV[s], &tmQKV, &kvfull[s], vcol, r);
-        tma_load_2d(sV[s] + OPND / 2, &tmQKV, &kvfull[s], vcol + 64, r);
+        if (!mbar_wait(&kempty[s], ph, abort_flag, err, CORA_DERR_TMA_WAIT)) break;
+        mbar_arrive_expect_tx(&kfull[s], OPND);
+        tma_load_2d(sK[s], &tmQKV, &kfull[s], kcol, r);
+        tma_load_2d(sK[s] + OPND / 2, &tmQKV, &kfull[s], kcol + 64, r);
+        if (!mbar_wait(&vempty[s], ph, abort_flag, err, CORA_DERR_TMA_WAIT)) break;
+        mbar_arrive_expect_tx(&vfull[s], OPND);
+        tma_load_2d(sV[s], &tmQKV, &vfull[s], vcol, r);
+        tma_load_2d(sV[s] + OPND / 2, &tmQKV, &vfull[s], vcol + 64, r);
       }
     }
   } else if (warp == 1) {
@@ -183,6 +192,7 @@ __global__ void __launch_bounds__(192, 1)
       auto issue_pv = [&](int jj) -> bool {
         const int s = jj & 1;
         if (!mbar_wait(&pfull[s], (jj >> 1) & 1, abort_flag, err, CORA_DERR_MMA_WAIT)) return false;
+        if (!mbar_wait(&vfull[s], (jj >> 1) & 1, abort_flag, err, CORA_DERR_MMA_WAIT)) return false;
         tc_fence_after();
         const uint32_t p_addr = smem_u32(sP[s]), v_addr = smem_u32(sV[s]);
 #pragma unroll
@@ -194,13 +204,13 @@ __global__ void __launch_bounds__(192, 1)
           umma_bf16(o_tmem, a, bd, IDESC_PV, (jj > 0 || k > 0) ? 1u : 0u);
         }
         umma_commit(&pdone[s]);
-        umma_commit(&kvempty[s]);
+        umma_commit(&vempty[s]);
         return true;
       };
       for (int j = 0; ok && j < n_kt; ++j) {
         const int s = j & 1;
         const uint32_t ph = (j >> 1) & 1;
-        if (!mbar_wait(&kvfull[s], ph, abort_flag, err, CORA_DERR_MMA_WAIT)) break;
+        if (!mbar_wait(&kfull[s], ph, abort_flag, err, CORA_DERR_MMA_WAIT)) break;
         if (!mbar_wait(&sfree[s], ph ^ 1u, abort_flag, err, CORA_DERR_MMA_WAIT)) break;
         tc_fence_after();
         const uint32_t k_addr = smem_u32(sK[s]);
@@ -211,6 +221,7 @@ __global__ void __launch_bounds__(192, 1)
           umma_bf16(d, sw128_kmajor_desc(q_addr + off), sw128_kmajor_desc(k_addr + off), IDESC_QK, k > 0);
         }
         umma_commit(&sfull[s]);
+        umma_commit(&kempty[s]);
         if (j >= 1 && !issue_pv(j - 1)) break;
       }
       if (ok && n_kt >= 1) issue_pv(n_kt - 1);
@@ -235,12 +246,18 @@ __global__ void __launch_bounds__(192, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfree[s]);  // S buffer may take S_{j+2}
       const int kbase = j * KT;
-      float mx = -INFINITY;
+      float mx8[8];
 #pragma unroll
-      for (int i = 0; i < KT; ++i) {
-        if (kbase + i >= S) v[i] = __float_as_uint(-INFINITY);
-        mx = fmaxf(mx, __uint_as_float(v[i]));
+      for (int i = 0; i < 8; ++i) mx8[i] = -INFINITY;
+      if (kbase + KT > S) {  // ragged last tile: keys past the end do not count
+#pragma unroll
+        for (int i = 0; i < KT; ++i)
+          if (kbase + i >= S) v[i] = __float_as_uint(-INFINITY);
       }
+#pragma unroll
+      for (int i = 0; i < KT; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(v[i]));  // eight chains
+      float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                       fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
       mx *= sl2;
       const bool raise = mx > m + kRescale;
       if (__any_sync(0xffffffffu, raise)) {
@@ -268,7 +285,7 @@ __global__ void __launch_bounds__(192, 1)
       // P buffer s is free once PV_{j-2} has read it.
       if (j >= 2) ok = mbar_wait(&pdone[s], ph ^ 1u, abort_flag, err, CORA_DERR_EPI_WAIT);
       if (!ok) break;
-      float rs = 0.f;
+      float rs4[4] = {0.f, 0.f, 0.f, 0.f};
       uint8_t* prow = sP[s];
 #pragma unroll
       for (int c = 0; c < KT; c += 8) {
@@ -277,7 +294,7 @@ __global__ void __launch_bounds__(192, 1)
         for (int i = 0; i < 4; ++i) {
           const float x0 = ex2f(fmaf(__uint_as_float(v[c + 2 * i]), sl2, -m));
           const float x1 = ex2f(fmaf(__uint_as_float(v[c + 2 * i + 1]), sl2, -m));
-          rs += x0 + x1;
+          rs4[i] += x0 + x1;
           pk[i] = pack_bf16x2(x0, x1);
         }
         // keys c .. c+7 -> swizzle column c/64, 16-byte chunk (c%64)/8
@@ -285,7 +302,7 @@ __global__ void __launch_bounds__(192, 1)
         *reinterpret_cast<uint4*>(prow + (c >> 6) * (OPND / 2) + r * 128 + ((chunk ^ (r & 7)) << 4)) =
             make_uint4(pk[0], pk[1], pk[2], pk[3]);
       }
-      l += rs;
+      l += (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
