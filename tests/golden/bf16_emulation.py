@@ -16,7 +16,7 @@ tests/test_gpu_kernels.py pins bit-exact to synth's host implementation
 (generating 8B parameters on the host takes over an hour).  This script
 computes no stored value and is not part of the test suite.
 
-    python tests/golden/bf16_emulation.py
+    python tests/golden/bf16_emulation.py [preset ...]
 """
 
 from __future__ import annotations
@@ -34,7 +34,7 @@ sys.path.insert(0, os.path.dirname(os.path.dirname(HERE)))
 
 from paper_2608_11235_gb300 import configs, model, synth  # noqa: E402
 
-PRESET = "llada8b-shape-256+256"
+PRESETS = ["llada8b-shape-256+256", "dream7b-shape-256+512-b4"]
 
 
 def bf(x: torch.Tensor) -> torch.Tensor:
@@ -82,7 +82,7 @@ def eq1(cfg: dict, xf: torch.Tensor):
     return prob.amax(-1).cpu().numpy(), prob.argmax(-1).cpu().numpy()
 
 
-def main() -> None:
+def main(PRESET: str) -> None:
     torch.backends.cuda.matmul.allow_tf32 = False
     base = configs.PRESETS[PRESET]
     P, G, BL, mask = base["prompt_len"], base["gen_len"], base["block_len"], base["mask_id"]
@@ -108,4 +108,5 @@ def main() -> None:
 
 
 if __name__ == "__main__":
-    main()
+    for p in sys.argv[1:] or PRESETS:
+        main(p)

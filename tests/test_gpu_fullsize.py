@@ -102,30 +102,40 @@ def check_heads(ref, c, a, head, label):
     print(f"{label}: max|dc| = {dc.max():.2e}, mean {dc.mean():.2e}, argmax on {int(sel.sum())}/32")
 
 
-def test_later_blocks_parity_full_size():
-    """The LLaDA-8B-shaped pass on seeded mid-decode canvases (blocks 1, 4, 7
-    at their first pass; blocks 3 and 6 with part of the block resolved),
-    set through cora_session_write, against stored oracle results."""
-    preset = PRESETS[0]
+BLOCK_PRESETS = [p for p in PRESETS if os.path.exists(os.path.join(GOLDEN, f"fullsize_{p}_blocks.json"))]
+
+
+@pytest.mark.parametrize("preset", BLOCK_PRESETS)
+def test_later_blocks_parity_full_size(preset):
+    """The workload's pass on seeded mid-decode canvases of sequence 0 (first
+    passes of later blocks; passes inside a block with part of it resolved),
+    set through cora_session_write in the batch the bench times (the other
+    sequences at their first step), against stored oracle results."""
     with open(os.path.join(GOLDEN, f"fullsize_{preset}_blocks.json")) as f:
         gold = json.load(f)
     base = configs.PRESETS[preset]
-    P, G, BL, T = base["prompt_len"], base["gen_len"], base["block_len"], base["steps_per_block"]
+    B, P, G, BL, T = base["batch"], base["prompt_len"], base["gen_len"], base["block_len"], base["steps_per_block"]
     for head, cfg in (("workload", base), ("gate_exercising", configs.gate_exercising(base))):
         m = model.create_model(cfg)
         try:
-            prompts = synth.prompts(cfg["prompt_seed"], 1, P, cfg["mask_id"])
-            s = cora.cora_session_create(m, 1, prompts, P, G, BL, T, cfg["tau"], cfg["K"])
+            prompts = synth.prompts(cfg["prompt_seed"], B, P, cfg["mask_id"])
+            s = cora.cora_session_create(m, B, prompts, P, G, BL, T, cfg["tau"], cfg["K"])
             try:
+                fresh = np.concatenate([prompts, np.full((B, G), cfg["mask_id"], np.int32)], axis=1)
                 for case in gold["cases"]:
                     blk = case["block"]
                     tokens, state = synth.mid_decode_canvas(cfg, case["canvas_seed"], blk, case["frac_resolved"])
                     step = int(state[blk * BL:(blk + 1) * BL].sum())  # any step < T; it only sets k
-                    cora.cora_session_write(s, tokens=tokens[None], state=state[None],
-                                            persist=np.zeros((1, BL), np.int32), prev=np.full((1, BL), -1, np.int32),
-                                            ctrl=np.array([[blk, min(step, T - 1), 0, 0]], np.int32))
+                    tok = fresh.copy()
+                    tok[0] = tokens
+                    st = np.zeros((B, G), np.uint8)
+                    st[0] = state
+                    ctrl = np.zeros((B, 4), np.int32)
+                    ctrl[0] = [blk, min(step, T - 1), 0, 0]
+                    cora.cora_session_write(s, tokens=tok, state=st, persist=np.zeros((B, BL), np.int32),
+                                            prev=np.full((B, BL), -1, np.int32), ctrl=ctrl)
                     cora.cora_denoise_step(s)
-                    out = cora.cora_session_read(s, 1, P + G, G, BL)
+                    out = cora.cora_session_read(s, B, P + G, G, BL)
                     check_heads(case["heads"][head], out["conf"][0], out["argmax"][0], head,
                                 f"{preset} block {blk} frac {case['frac_resolved']} [{head}]")
             finally:
