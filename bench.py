@@ -42,12 +42,13 @@ import numpy as np  # noqa: E402
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM bytes (read + write) per launch from one ncu capture of each kernel on
-# the LLaDA-8B-shaped workload (2-layer model, same per-launch shapes), keyed
-# by a hash of the kernel source at capture time; null once the source changed.
+# a workload's per-launch shapes (2-layer model), keyed by a hash of the
+# kernel source at capture time and by the workload; null once the source
+# changed, and for workloads without a capture.
 NCU_TRAFFIC = {
     # gemm_tc2_kernel, mean of the QKV / O / gate-up / down launches (read + write):
     # (126.0 + 46.3 + 246.3 + 125.5) MB / 4, profiles/gemm_tc2_llada8b_256.md
-    ("gemm", "2f06f7bcf379"): 136_028_000,
+    ("gemm", "2f06f7bcf379", "llada8b-shape-256+256"): 136_028_000,
 }
 
 
@@ -342,7 +343,7 @@ def run_cora(args, cfg, ws, rank, local):
     attn_ms = sum(by["attention"]) / len(by["attention"])
     kernels = {k: {"launches_per_pass": len(v), "ms_per_launch": round(sum(v) / len(v), 5),
                    "share": round(sum(v) / step_ms, 4)} for k, v in sorted(by.items())}
-    traffic = NCU_TRAFFIC.get(("gemm", src_hash("gemm.cu")))
+    traffic = NCU_TRAFFIC.get(("gemm", src_hash("gemm.cu"), cfg["name"]))  # per workload: the shapes differ
     roofline = {"bound": "tensor", "kernel": "gemm_tc2_kernel (QKV+RoPE, O+res, gate/up+SwiGLU, down+res)",
                 "achieved": round(gemm_tflops, 2), "peak": peak_tf, "unit": "TFLOP/s",
                 "frac": round(gemm_tflops / peak_tf, 4), "traffic": traffic,
