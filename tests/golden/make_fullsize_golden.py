@@ -17,7 +17,8 @@ probability margin and logit gap per row, for each head).
 Later blocks: the same pass on seeded mid-decode canvases of sequence 0
 (synth.mid_decode_canvas), per workload in BLOCK_CASES: first passes of
 later blocks and passes inside a block with part of it already resolved.
-Output: tests/golden/fullsize_<preset>_blocks.json.
+Output: tests/golden/fullsize_<preset>_blocks.json (cases already there are
+kept, so new cases can be added without recomputing the others).
 """
 
 from __future__ import annotations
@@ -55,7 +56,8 @@ def head_eq1(cfg, rows, v_chunk=16384):
 CANVAS_SEED = 500
 # (active block, fraction of it already resolved) per workload
 BLOCK_CASES = {
-    "llada8b-shape-256+256": [(1, 0.0), (4, 0.0), (7, 0.0), (3, 0.5), (6, 0.75)],
+    "llada8b-shape-256+256": [(1, 0.0), (4, 0.0), (7, 0.0), (3, 0.5), (6, 0.75), (2, 0.0), (3, 0.0), (5, 0.0),
+                              (6, 0.0)],
     "dream7b-shape-256+512-b4": [(5, 0.0), (15, 0.0), (10, 0.5)],
     "llada8b-shape-512+1024-b8": [(15, 0.0), (31, 0.0)],
 }
@@ -74,9 +76,20 @@ def forward_rows(cfg, tokens, block, tag):
 
 
 def run_blocks(preset: str) -> None:
+    """Cases already in the output file (same canvas seed) are kept, not recomputed."""
     cfg = dict(configs.PRESETS[preset])
+    path = os.path.join(HERE, f"fullsize_{preset}_blocks.json")
+    done = {}
+    if os.path.exists(path):
+        with open(path) as f:
+            for c in json.load(f)["cases"]:
+                if c["canvas_seed"] == CANVAS_SEED:
+                    done[(c["block"], c["frac_resolved"])] = c
     cases = []
     for block, frac in BLOCK_CASES[preset]:
+        if (block, frac) in done:
+            cases.append(done[(block, frac)])
+            continue
         tokens, state = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, frac)
         rows = forward_rows(cfg, tokens, block, f"{preset} block {block} frac {frac}")
         cases.append({"block": block, "frac_resolved": frac, "canvas_seed": CANVAS_SEED,
@@ -85,7 +98,7 @@ def run_blocks(preset: str) -> None:
     out = {"preset": preset, "sequence": 0,
            "source": "oracle/cora_oracle.py (layer_forward, lm_logits, top1, top2_margin), float64",
            "cases": cases}
-    with open(os.path.join(HERE, f"fullsize_{preset}_blocks.json"), "w") as f:
+    with open(path, "w") as f:
         json.dump(out, f)
 
 
