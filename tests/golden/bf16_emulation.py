@@ -34,7 +34,7 @@ sys.path.insert(0, os.path.dirname(os.path.dirname(HERE)))
 
 from paper_2608_11235_gb300 import configs, model, synth  # noqa: E402
 
-PRESETS = ["llada8b-shape-256+256", "dream7b-shape-256+512-b4"]
+PRESETS = ["llada8b-shape-256+256", "dream7b-shape-256+512-b4", "llada8b-shape-512+1024-b8"]
 
 
 def bf(x: torch.Tensor) -> torch.Tensor:
