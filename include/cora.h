@@ -398,6 +398,19 @@ CORA_API int cora_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, 
  * the current device: 0 when no kernel has recorded a fault. */
 CORA_API int cora_device_error(int32_t* code, int32_t clear);
 
+/* Failure-detection self-check (every wait in the kernels is bounded, and an
+ * expired wait is reported, not fatal).  Launches one CTA on the current device
+ * whose thread waits, with the kernels' own bounded waits, on an mbarrier
+ * that nothing arrives at (which = 0) or on a global flag that nothing sets
+ * (which = 1).  The wait gives up after the library's limit (~2 s), the
+ * kernel records its code in a fresh error word of its own and returns; the
+ * call synchronises the device and writes that word to *code_out (0x102 for
+ * the mbarrier, 0x104 for the flag).  The context stays usable; the
+ * library's device error word is not touched.  Allocates 8 bytes of device
+ * memory for the duration of the call.  Errors: CORA_EINVAL for a bad
+ * argument or NULL code_out, CORA_ECUDA if a CUDA call fails. */
+CORA_API int cora_check_wait_timeout(int32_t which, int32_t* code_out);
+
 #ifdef __cplusplus
 }
 #endif

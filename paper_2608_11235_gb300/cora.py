@@ -26,7 +26,7 @@ EXPORTED = [
     "cora_session_batched_passes", "cora_generate", "cora_gate_transfer", "cora_reduce_top1", "cora_reduce_gate",
     "cora_op_gemm", "cora_op_attention", "cora_op_rmsnorm", "cora_op_lm_head_top1", "cora_synth_normal_bf16",
     "cora_device_error", "cora_session_profile_step", "cora_session_stream", "cora_reduce_top1_noalloc",
-    "cora_session_create_ex", "cora_generate_ex", "cora_session_disagreement",
+    "cora_session_create_ex", "cora_generate_ex", "cora_session_disagreement", "cora_check_wait_timeout",
 ]
 SCHEDULE_FIXED, SCHEDULE_REMAINING = 0, 1
 PERSIST_BLOCK, PERSIST_CARRY = 0, 1
@@ -109,6 +109,7 @@ def lib():
             "cora_op_lm_head_top1": ([vp, vp, i32, i32, i32, vp, vp, vp], C.c_int),
             "cora_synth_normal_bf16": ([vp, i64, u64, i64, f32, vp], C.c_int),
             "cora_device_error": ([vp, i32], C.c_int),
+            "cora_check_wait_timeout": ([i32, vp], C.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -323,6 +324,14 @@ def cora_op_lm_head_top1(x, W, R, V, d, conf, argmax, stream=None) -> None:
 def cora_synth_normal_bf16(out, count, key, start, scale, stream=None) -> None:
     _check("cora_synth_normal_bf16", lib().cora_synth_normal_bf16(ptr(out), count, key, start, float(scale),
                                                                   _stream(stream)))
+
+
+def cora_check_wait_timeout(which: int) -> int:
+    """Runs the bounded-wait self-check (0: an mbarrier nothing arrives at, 1: a
+    flag nothing sets); returns the error code the kernel recorded."""
+    code = np.zeros(1, np.int32)
+    _check("cora_check_wait_timeout", lib().cora_check_wait_timeout(int(which), ptr(code)))
+    return int(code[0])
 
 
 def cora_device_error(clear: bool = False) -> int:

@@ -166,6 +166,8 @@ bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t
                        uint64_t stride2_bytes, uint32_t b0, uint32_t b1, uint32_t b2);
 
 int gemm_block_n(int N, int mode);
+// Failure-detection self-check (see cora_check_wait_timeout).
+cudaError_t launch_wait_check(int which, const int* flag, int* err, cudaStream_t st);
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,
                         const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st);
 bool make_gemm_out_tmap(CUtensorMap* map, void* C, int M, int ldc, int mode);

@@ -1114,6 +1114,33 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
 
 }  // namespace cora
 
+namespace cora {
+
+// Failure-detection self-check: one thread waits, with the same bounded waits
+// as the GEMM's pipeline, on an mbarrier that nothing arrives at (which = 0)
+// or on a flag that nothing sets (which = 1); the wait gives up after
+// CORA_WAIT_LIMIT cycles, records its code in `err` and the kernel returns.
+__global__ void wait_check_kernel(int which, const int* flag, int* err) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    volatile int* ab = &abort_flag;
+    if (which == 0)
+      (void)mbar_wait(&bar, 0, ab, err, CORA_DERR_MMA_WAIT);  // phase 0 never completes
+    else
+      (void)wait_flag(flag, ab, err);  // *flag stays 0
+  }
+  __syncthreads();
+}
+
+}  // namespace cora
+
 using namespace cora;
 
 // The 2-CTA kernel is used for M > 128 unless switched off (cora_gemm_pairs).
@@ -1186,6 +1213,11 @@ static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB
 // and half the SMs.
 static int gemm2_pairs(int M, int N, int K, int num_sms, GemmEpilogue& ep) {
   return gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2, ep);
+}
+
+cudaError_t launch_wait_check(int which, const int* flag, int* err, cudaStream_t st) {
+  wait_check_kernel<<<1, 32, 0, st>>>(which, flag, err);
+  return cudaGetLastError();
 }
 
 cudaError_t gemm_prepare() {

@@ -1104,6 +1104,24 @@ extern "C" int cora_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key
   return CORA_OK;
 }
 
+extern "C" int cora_check_wait_timeout(int32_t which, int32_t* code_out) {
+  REQUIRE(code_out && (which == 0 || which == 1), "cora_check_wait_timeout: bad argument");
+  DeviceCtx* dc = nullptr;
+  int rc = device_ctx(&dc);
+  if (rc) return rc;
+  int* buf = nullptr;  // [0] the flag nothing sets, [1] this check's own error word
+  CK(cudaMalloc(&buf, 2 * sizeof(int)));
+  cudaError_t e = cudaMemset(buf, 0, 2 * sizeof(int));
+  if (e == cudaSuccess) e = launch_wait_check(which, buf, buf + 1, 0);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  int code = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&code, buf + 1, sizeof(int), cudaMemcpyDeviceToHost);
+  cudaFree(buf);
+  CK(e);
+  *code_out = code;
+  return CORA_OK;
+}
+
 extern "C" int cora_device_error(int32_t* code, int32_t clear) {
   REQUIRE(code, "cora_device_error: NULL pointer");
   DeviceCtx* dc = nullptr;

@@ -210,3 +210,17 @@ def test_reduce_top1(rows, V):
     arg.zero_()
     cora.cora_reduce_top1(lg_dev, rows, V, conf, arg)   # second call: completion counters were left at zero
     assert np.array_equal(conf.cpu().numpy(), c) and np.array_equal(arg.cpu().numpy(), a)
+
+
+# ----------------------------------------------------------- failure detection
+@pytest.mark.parametrize("which,code", [(0, 0x102), (1, 0x104)])
+def test_bounded_wait_reports_and_context_survives(which, code):
+    """A wait that nothing completes (an mbarrier nobody arrives at, a flag
+    nobody sets) gives up after the kernels' limit and reports its code; the
+    context then runs a normal kernel."""
+    assert cora.cora_check_wait_timeout(which) == code
+    x = f64(bits(9, 1, (4, 256), 1.0)).astype(np.float32)
+    out = torch.empty((4, 256), dtype=torch.int16, device="cuda")
+    cora.cora_op_rmsnorm(torch.from_numpy(x).cuda(), None, out, 4, 256, 1e-5)
+    close_bf16(from_dev_bf16(out), O.rms_norm(x.astype(np.float64), np.ones(256), 1e-5))
+    assert cora.cora_device_error() == 0
