@@ -416,3 +416,49 @@ def test_prefix_cache_batch_moves_blocks_together(sharp):
         print(f"prefix-cache batch: {waited} waiting sequence-steps, passes {active_steps.tolist()}")
     finally:
         cora.cora_session_destroy(s)
+
+
+@pytest.mark.parametrize("frac", [0.05, 0.5, 0.9])
+def test_checkpoint_and_resume_in_a_new_session(sharp, frac):
+    """Checkpoint/resume at step granularity: a decode stopped after some
+    steps, its state read out (canvas, position states, persistence, previous
+    predictions, block/step/pass counters) and written into a fresh session
+    continues to the same tokens and pass counts as an uninterrupted decode
+    (the kernels are deterministic, so equality is exact)."""
+    m, prompt = sharp
+    B = prompt.shape[0]
+    cfg = dict(configs.TINY_SHARP)
+    tau, Kp = cfg["tau"], cfg["K"]
+
+    def run_to_end(s):
+        n = 1
+        while not cora.cora_denoise_step(s):
+            n += 1
+            assert n <= (G // BL) * T
+        return cora.cora_session_read(s, B, P + G, G, BL), n
+
+    s = cora.cora_session_create(m, B, prompt, P, G, BL, T, tau, Kp)
+    try:
+        ref, n_steps = run_to_end(s)
+    finally:
+        cora.cora_session_destroy(s)
+    stop_after = max(1, min(n_steps - 1, int(frac * n_steps)))
+    s = cora.cora_session_create(m, B, prompt, P, G, BL, T, tau, Kp)
+    try:
+        for _ in range(stop_after):
+            assert not cora.cora_denoise_step(s)
+        ck = cora.cora_session_read(s, B, P + G, G, BL)
+    finally:
+        cora.cora_session_destroy(s)
+    s = cora.cora_session_create(m, B, prompt, P, G, BL, T, tau, Kp)
+    try:
+        cora.cora_session_write(s, tokens=ck["tokens"], state=ck["state"], persist=ck["persist"], prev=ck["prev"],
+                                ctrl=ck["ctrl"])
+        out, n_rest = run_to_end(s)
+    finally:
+        cora.cora_session_destroy(s)
+    assert stop_after + n_rest == n_steps
+    assert np.array_equal(out["tokens"], ref["tokens"])
+    assert np.array_equal(out["state"], ref["state"])
+    assert np.array_equal(out["ctrl"], ref["ctrl"])  # block, step, passes executed, finished
+    assert cora.cora_device_error() == 0
