@@ -152,14 +152,16 @@ def test_later_blocks_parity_full_size(preset):
 GATE_BLOCKS = {"llada8b-shape-256+256": None, "dream7b-shape-256+512-b4": None, "llada8b-shape-512+1024-b8": 4}
 
 
+@pytest.mark.parametrize("schedule", ["fixed", "remaining"])
 @pytest.mark.parametrize("preset", PRESETS)
-def test_gate_every_step_full_size(preset):
+def test_gate_every_step_full_size(preset, schedule):
     """Eq. 2-4 and block termination, bit-exact at every executed step of the
     full-size decode: before each cora_denoise_step the session's state is
     read; the oracle's step (oracle.cora_step) is applied to that state with
     the GPU's own Eq. 1 outputs (float32 confidence, argmax) of the step; its
     transfer and acceptance sets, canvas, position states, persistence and
-    control must equal the GPU's.  Gate-exercising head, so the gate fires."""
+    control must equal the GPU's.  Gate-exercising head, so the gate fires;
+    the fixed schedule and the remaining-steps one (k = ceil(|U| / (T - s)))."""
     from oracle import cora_oracle as O
     cfg = configs.gate_exercising(configs.PRESETS[preset])
     B, P, G, BL, T = cfg["batch"], cfg["prompt_len"], cfg["gen_len"], cfg["block_len"], cfg["steps_per_block"]
@@ -171,7 +173,8 @@ def test_gate_every_step_full_size(preset):
     m = model.create_model(cfg)
     steps = accepted = blocks_done = 0
     try:
-        s = cora.cora_session_create(m, B, prompts, P, G, BL, T, tau, K)
+        opts = cora.decode_options(schedule=cora.SCHEDULE_REMAINING) if schedule == "remaining" else None
+        s = cora.cora_session_create(m, B, prompts, P, G, BL, T, tau, K, options=opts)
         try:
             before = cora.cora_session_read(s, B, P + G, G, BL)
             while np.any(before["ctrl"][:, 0] < stop_block):
@@ -186,7 +189,9 @@ def test_gate_every_step_full_size(preset):
                     st = O.BlockState(before["tokens"][b, p0:p0 + BL].astype(np.int64),
                                       before["state"][b, g0:g0 + BL].copy(),
                                       before["persist"][b].astype(np.int64), before["prev"][b].astype(np.int64))
-                    r = O.cora_step(st, after["conf"][b], after["argmax"][b].astype(np.int64), ks[step], tau, K)
+                    k = (O.remaining_step_count(int((st.state == O.UNRESOLVED).sum()), T, step)
+                         if schedule == "remaining" else ks[step])
+                    r = O.cora_step(st, after["conf"][b], after["argmax"][b].astype(np.int64), k, tau, K)
                     lbl = (preset, b, blk, step)
                     assert sorted(np.flatnonzero(after["unmask"][b])) == r.transferred, lbl
                     assert sorted(np.flatnonzero(after["accept"][b])) == r.accepted, lbl
@@ -211,4 +216,82 @@ def test_gate_every_step_full_size(preset):
         cora.cora_model_destroy(m)
         torch.cuda.empty_cache()
     assert accepted > 0 and blocks_done >= B
-    print(f"{preset}: {steps} sequence-steps checked, {blocks_done} blocks ended, {accepted} positions accepted")
+    print(f"{preset} [{schedule}]: {steps} sequence-steps checked, {blocks_done} blocks ended, "
+          f"{accepted} positions accepted")
+
+
+CACHED_PRESETS = [p for p in PRESETS if os.path.exists(os.path.join(GOLDEN, f"fullsize_{p}_cached.json"))]
+
+
+@pytest.mark.parametrize("preset", CACHED_PRESETS)
+def test_prefix_cache_pass_full_size(preset):
+    """The prefix-cache step (a decoding variant) at full size: a session with
+    the prefix cache runs the block's dense first pass on the canvas with the
+    block fully masked (keeping every layer's keys/values), then, set through
+    cora_session_write to the same canvas with part of the block resolved, a
+    cached pass over the rows from the block's start on; Eq. 1 of that pass
+    against the stored oracle results (same tolerances as the later blocks)."""
+    with open(os.path.join(GOLDEN, f"fullsize_{preset}_cached.json")) as f:
+        gold = json.load(f)
+    base = configs.PRESETS[preset]
+    B, P, G, BL, T = base["batch"], base["prompt_len"], base["gen_len"], base["block_len"], base["steps_per_block"]
+    for head, cfg in (("workload", base), ("gate_exercising", configs.gate_exercising(base))):
+        m = model.create_model(cfg)
+        try:
+            prompts = synth.prompts(cfg["prompt_seed"], B, P, cfg["mask_id"])
+            s = cora.cora_session_create(m, B, prompts, P, G, BL, T, cfg["tau"], cfg["K"],
+                                         options=cora.decode_options(cache=cora.CACHE_PREFIX))
+            try:
+                for case in gold["cases"]:
+                    blk = case["block"]
+                    for frac, step in ((0.0, 0), (case["frac_resolved"], 1)):  # step 0: dense; later: cached
+                        tokens, state = synth.mid_decode_canvas(cfg, case["canvas_seed"], blk, frac)
+                        cora.cora_session_write(s, tokens=tokens[None], state=state[None],
+                                                persist=np.zeros((B, BL), np.int32),
+                                                prev=np.full((B, BL), -1, np.int32),
+                                                ctrl=np.array([[blk, step, 0, 0]], np.int32))
+                        cora.cora_denoise_step(s)
+                    out = cora.cora_session_read(s, B, P + G, G, BL)
+                    check_heads(case["heads"][head], out["conf"][0], out["argmax"][0], head,
+                                f"{preset} cached pass, block {blk} frac {case['frac_resolved']} [{head}]")
+            finally:
+                cora.cora_session_destroy(s)
+            assert cora.cora_device_error() == 0
+        finally:
+            cora.cora_model_destroy(m)
+            torch.cuda.empty_cache()
+
+
+def test_disagreement_full_size():
+    """L^acc / L^out at full size (LLaDA-8B shape, gate-exercising head): the
+    session's counts against the definitions applied on the host to the
+    gated and the dense (gate off) decodes' canvases; integer counts, exact."""
+    from oracle import cora_oracle as O
+    preset = PRESETS[0]
+    cfg = configs.gate_exercising(configs.PRESETS[preset])
+    B, P, G, BL, T = cfg["batch"], cfg["prompt_len"], cfg["gen_len"], cfg["block_len"], cfg["steps_per_block"]
+    prompts = synth.prompts(cfg["prompt_seed"], B, P, cfg["mask_id"])
+    m = model.create_model(cfg)
+    try:
+        s = cora.cora_session_create(m, B, prompts, P, G, BL, T, cfg["tau"], cfg["K"])
+        d = cora.cora_session_create(m, B, prompts, P, G, BL, T, 2.0, 1)  # gate off: the dense endpoint
+        try:
+            cora.cora_session_run(s)
+            cora.cora_session_run(d)
+            n_acc, n_ad, n_od = cora.cora_session_disagreement(s, d, B)
+            a = cora.cora_session_read(s, B, P + G, G, BL)
+            ref = cora.cora_session_read(d, B, P + G, G, BL)["tokens"][:, P:]
+            for b in range(B):
+                tok, st = a["tokens"][b, P:], a["state"][b]
+                l_acc, l_out = O.disagreement(tok, st, ref[b])
+                assert n_acc[b] == int((st == O.ACCEPTED).sum()) > 0
+                assert l_acc == n_ad[b] / max(1, n_acc[b]) and l_out == n_od[b] / G
+            print(f"{preset}: {int(n_acc[0])} accepted, L_acc = {n_ad[0] / max(1, n_acc[0]):.3f}, "
+                  f"L_out = {n_od[0] / G:.3f}")
+        finally:
+            cora.cora_session_destroy(s)
+            cora.cora_session_destroy(d)
+        assert cora.cora_device_error() == 0
+    finally:
+        cora.cora_model_destroy(m)
+        torch.cuda.empty_cache()
