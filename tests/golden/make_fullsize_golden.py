@@ -19,6 +19,16 @@ Later blocks: the same pass on seeded mid-decode canvases of sequence 0
 later blocks and passes inside a block with part of it already resolved.
 Output: tests/golden/fullsize_<preset>_blocks.json (cases already there are
 kept, so new cases can be added without recomputing the others).
+
+    python tests/golden/make_fullsize_golden.py --cached [preset ...]
+
+Prefix-cache step (a decoding variant), per workload in CACHED_CASES: the
+dense pass on the canvas with the active block fully masked keeps every
+layer's keys/values; the pass on the same canvas with part of the block
+resolved recomputes the rows from the block's start on, the positions before
+it contributing their kept keys/values (the oracle's layer_forward_prefix,
+layer by layer for both canvases, as forward_hidden_kv and
+forward_hidden_cached compose it).  Output: tests/golden/fullsize_<preset>_cached.json.
 """
 
 from __future__ import annotations
@@ -102,6 +112,41 @@ def run_blocks(preset: str) -> None:
         json.dump(out, f)
 
 
+CACHED_CASES = {"llada8b-shape-256+256": [(3, 0.5), (6, 0.75)]}  # (block, fraction resolved at the cached pass)
+
+
+def run_cached(preset: str) -> None:
+    cfg = dict(configs.PRESETS[preset])
+    P, BL = cfg["prompt_len"], cfg["block_len"]
+    hkv, hd = cfg["n_kv_heads"], cfg["head_dim"]
+    cases = []
+    for block, frac in CACHED_CASES[preset]:
+        tok_a, _ = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, 0.0)   # the block's first pass
+        tok_b, _ = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, frac)  # a later pass of the block
+        lo = P + block * BL
+        assert np.array_equal(tok_a[:lo], tok_b[:lo])
+        embed = lambda toks: np.stack([synth.weight_f64(cfg, -1, synth.EMBED, slice(int(t), int(t) + 1))[0]
+                                       for t in toks])
+        ha, hb = embed(tok_a), embed(tok_b[lo:])
+        pos = np.arange(len(tok_a))
+        empty = np.zeros((0, hkv, hd))
+        t0 = time.time()
+        for l in range(cfg["n_layers"]):
+            lw = synth.layer_weights_f64(cfg, l)
+            ha, k, v = O.layer_forward_prefix(cfg, lw, ha, pos, empty, empty)
+            hb, _, _ = O.layer_forward_prefix(cfg, lw, hb, pos[lo:], k[:lo], v[:lo])
+            print(f"{preset} cached block {block} frac {frac}: layer {l} done at {time.time() - t0:.0f} s", flush=True)
+        rows = hb[:BL]
+        cases.append({"block": block, "frac_resolved": frac, "canvas_seed": CANVAS_SEED,
+                      "heads": {"workload": head_eq1(cfg, rows),
+                                "gate_exercising": head_eq1(configs.gate_exercising(cfg), rows)}})
+    out = {"preset": preset, "sequence": 0,
+           "source": "oracle/cora_oracle.py (layer_forward_prefix, lm_logits, top1, top2_margin), float64",
+           "cases": cases}
+    with open(os.path.join(HERE, f"fullsize_{preset}_cached.json"), "w") as f:
+        json.dump(out, f)
+
+
 def run(preset: str) -> None:
     cfg = dict(configs.PRESETS[preset])
     P, G, BL = cfg["prompt_len"], cfg["gen_len"], cfg["block_len"]
@@ -127,6 +172,9 @@ if __name__ == "__main__":
     if args and args[0] == "--blocks":
         for p in (args[1:] or PRESETS[:1]):
             run_blocks(p)
+    elif args and args[0] == "--cached":
+        for p in (args[1:] or PRESETS[:1]):
+            run_cached(p)
     else:
         for p in (args or PRESETS):
             run(p)
