@@ -206,6 +206,38 @@ def kernel_costs(cfg: dict):
     }
 
 
+def tiny_leg(reps: int = 5):
+    """The tiny two-layer model at its own operating point (tau 0.9, K 2): GPU
+    decode rate through cora_generate (device loop), passes per block, and the
+    oracle's whole decode of the same prompt timed on the host (numpy float64,
+    the library's default thread count)."""
+    import time as _t
+
+    from oracle import cora_oracle as O
+    from paper_2608_11235_gb300 import configs, cora, model, synth
+
+    cfg = dict(configs.TINY)
+    P, G, BL, T = cfg["prompt_len"], cfg["gen_len"], cfg["block_len"], cfg["steps_per_block"]
+    prompt = synth.prompts(cfg["prompt_seed"], 1, P, cfg["mask_id"])
+    m = model.create_model(cfg)
+    try:
+        cora.cora_generate(m, prompt, G, BL, T, cfg["tau"], cfg["K"])  # warm (graph capture)
+        t0 = _t.perf_counter()
+        for _ in range(reps):
+            _, passes, _ = cora.cora_generate(m, prompt, G, BL, T, cfg["tau"], cfg["K"])
+        gpu_s = (_t.perf_counter() - t0) / reps
+    finally:
+        cora.cora_model_destroy(m)
+    w = synth.model_weights_f64(cfg)
+    t0 = _t.perf_counter()
+    tr = O.generate(cfg, w, prompt[0], G, BL, T, cfg["tau"], cfg["K"])
+    ora_s = _t.perf_counter() - t0
+    return {"workload": cfg["name"], "tokens_per_s": round(G / gpu_s, 2), "passes": int(passes[0]),
+            "passes_per_block": round(float(passes[0]) / (G // BL), 2), "timing": "host wall clock, cora_generate",
+            "oracle_generate_s": round(ora_s, 3), "oracle_passes": int(sum(tr.passes_per_block)),
+            "oracle_tokens_per_s": round(G / ora_s, 2)}
+
+
 def gate_isolation(peaks, reps: int = 5):
     """Eq. 1 from materialised bf16 logits [B, 32, 126464] + transfer rule +
     gate (cora_reduce_gate), B in {1, 8, 64}; HBM-bound.  L2 is flushed
@@ -422,6 +454,7 @@ def run_cora(args, cfg, ws, rank, local):
         cora.cora_session_destroy(s)
     cora.cora_model_destroy(m)
     gate_iso = None if args.no_variant else gate_isolation(peaks)
+    tiny = None if args.no_variant else tiny_leg()
 
     value = ws * B * G * args.steps / (ms * 1e-3)
     # embed, final norm, LM head, gate + per layer 2 RMSNorms, 4 GEMMs, attention; the device
@@ -453,6 +486,7 @@ def run_cora(args, cfg, ws, rank, local):
         "gate_exercising": gx,
         "prefix_cache": pc,
         "gate_isolation": gate_iso,
+        "tiny": tiny,
     }
     return result, float(per_seq_passes.mean())
 
