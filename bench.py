@@ -47,8 +47,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # changed, and for workloads without a capture.
 NCU_TRAFFIC = {
     # gemm_tc2_kernel, mean of the QKV / O / gate-up / down launches (read + write):
-    # (126.0 + 46.3 + 246.3 + 125.5) MB / 4, profiles/gemm_tc2_llada8b_256.md
-    ("gemm", "2f06f7bcf379", "llada8b-shape-256+256"): 136_028_000,
+    # (124.4 + 46.3 + 245.1 + 125.6) MB / 4, profiles/gemm_tc2_llada8b_256.md
+    ("gemm", "d8e0704d8d40", "llada8b-shape-256+256"): 135_355_000,
 }
 
 
