@@ -68,8 +68,9 @@ CANVAS_SEED = 500
 BLOCK_CASES = {
     "llada8b-shape-256+256": [(1, 0.0), (4, 0.0), (7, 0.0), (3, 0.5), (6, 0.75), (2, 0.0), (3, 0.0), (5, 0.0),
                               (6, 0.0)],
-    "dream7b-shape-256+512-b4": [(5, 0.0), (15, 0.0), (10, 0.5)],
-    "llada8b-shape-512+1024-b8": [(15, 0.0), (31, 0.0)],
+    "dream7b-shape-256+512-b4": [(5, 0.0), (15, 0.0), (10, 0.5)] + [(b, 0.0) for b in (1, 2, 3, 4, 6, 7, 8, 9, 11, 12,
+                                                                                 13, 14)] + [(3, 0.25), (12, 0.75)],
+    "llada8b-shape-512+1024-b8": [(15, 0.0), (31, 0.0), (7, 0.5), (23, 0.75)],
 }
 
 
