@@ -238,11 +238,14 @@ def tiny_leg(reps: int = 5):
             "oracle_tokens_per_s": round(G / ora_s, 2)}
 
 
-def gate_isolation(peaks, reps: int = 5):
+def gate_isolation(peaks, reps: int = 5, with_oracle: bool = False):
     """Eq. 1 from materialised bf16 logits [B, 32, 126464] + transfer rule +
     gate (cora_reduce_gate), B in {1, 8, 64}; HBM-bound.  L2 is flushed
     (a 256 MB write) before every timed launch; CUDA events bracket the launch
-    only."""
+    only.  With ``with_oracle`` the oracle's reduction + gate on the same
+    logits and state is timed on the host as the CPU baseline (float64 numpy,
+    the library's default thread count; the bf16 -> float32 widening of the
+    logits is outside the timing)."""
     import torch
 
     from paper_2608_11235_gb300 import configs, cora, synth
@@ -253,7 +256,8 @@ def gate_isolation(peaks, reps: int = 5):
     out = {}
     for B in gi["batches"]:
         hist = synth.gate_history(gi["seed"], B, R, V, gi["n_hist"], gi["keep"])
-        lg = torch.from_numpy(synth.gate_logits_bf16(gi["seed"], B, R, V, hist[-1], gi["keep"]).view(np.int16)).cuda()
+        lg_host = synth.gate_logits_bf16(gi["seed"], B, R, V, hist[-1], gi["keep"])
+        lg = torch.from_numpy(lg_host.view(np.int16)).cuda()
         st = lambda dt: torch.zeros((B, R), dtype=dt, device="cuda")
         conf, arg, prev, persist = st(torch.float32), st(torch.int32), st(torch.int32), st(torch.int32)
         state, tokens, unmask, accept = st(torch.uint8), st(torch.int32), st(torch.uint8), st(torch.uint8)
@@ -278,6 +282,56 @@ def gate_isolation(peaks, reps: int = 5):
         out[f"B{B}"] = {"us": round(ms * 1e3, 2), "GB_s": round(gbs, 1),
                         "frac": round(gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]), 4), "bytes": nbytes}
         del lg
+        if with_oracle:
+            from oracle import cora_oracle as O
+            lf = synth.bf16_bits_to_f32(lg_host)
+            z = np.zeros((B, R), np.int64)
+            t0 = time.perf_counter()
+            O.reduce_and_gate(lf, z, z.astype(np.uint8), z, np.full((B, R), -1, np.int64), gi["k_step"], gi["tau"],
+                              gi["K"])
+            dt = time.perf_counter() - t0
+            out[f"B{B}"]["cpu_baseline"] = {"kind": "oracle", "us": round(dt * 1e6, 1),
+                                            "GB_s": round(nbytes / dt / 1e9, 3)}
+    return out
+
+
+def attention_shapes(peaks, reps: int = 5):
+    """The attention kernel alone at the attention shape of each 8B-class
+    workload (batch, canvas length, heads as configured; seeded N(0, 1) bf16
+    Q/K/V from the device generator).  FLOPs per launch 4 B Hq S^2 hd against
+    the burst bf16 peak (a kernel timed in isolation).  L2 is flushed (a 256 MB
+    write) before every timed launch; CUDA events bracket the launch only."""
+    import torch
+
+    from paper_2608_11235_gb300 import configs, cora, synth
+
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    out = {}
+    for name in ("llada8b-shape-256+256", "dream7b-shape-256+512-b4", "llada8b-shape-512+1024-b8"):
+        c = configs.PRESETS[name]
+        B, S = c["batch"], c["prompt_len"] + c["gen_len"]
+        hq, hkv, hd = c["n_heads"], c["n_kv_heads"], c["head_dim"]
+        n = B * S * (hq + 2 * hkv) * hd
+        qkv = torch.empty(n, dtype=torch.int16, device="cuda")
+        o = torch.empty(B * S * hq * hd, dtype=torch.int16, device="cuda")
+        cora.cora_synth_normal_bf16(qkv, n, synth.stream_key(23, 1), 0, float(synth.normal_scale_f32(1.0)))
+        ts = []
+        for i in range(reps + 2):
+            flush.fill_(i & 0xFF)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            cora.cora_op_attention(qkv, o, B, S, hq, hkv, hd)
+            e1.record()
+            e1.synchronize()
+            if i >= 2:
+                ts.append(e0.elapsed_time(e1))
+        ms = statistics.median(ts)
+        tf = 4.0 * B * hq * S * S * hd / (ms * 1e-3) / 1e12
+        out[name] = {"B": B, "S": S, "Hq": hq, "Hkv": hkv, "hd": hd, "us": round(ms * 1e3, 2),
+                     "achieved": round(tf, 1), "unit": "TFLOP/s", "peak": peak, "frac": round(tf / peak, 4)}
+        del qkv, o
+    out["peak_source"] = "bf16 burst (kernel timed alone)"
     return out
 
 
@@ -453,8 +507,10 @@ def run_cora(args, cfg, ws, rank, local):
     if s is not None:
         cora.cora_session_destroy(s)
     cora.cora_model_destroy(m)
-    gate_iso = None if args.no_variant else gate_isolation(peaks)
+    gate_iso = None if args.no_variant else gate_isolation(
+        peaks, with_oracle=(rank == 0 and ws == 1 and not args.no_cpu_baseline))
     tiny = None if args.no_variant else tiny_leg()
+    attn_shapes = None if args.no_variant else attention_shapes(peaks)
 
     value = ws * B * G * args.steps / (ms * 1e-3)
     # embed, final norm, LM head, gate + per layer 2 RMSNorms, 4 GEMMs, attention; the device
@@ -487,6 +543,7 @@ def run_cora(args, cfg, ws, rank, local):
         "prefix_cache": pc,
         "gate_isolation": gate_iso,
         "tiny": tiny,
+        "attention_shapes": attn_shapes,
     }
     return result, float(per_seq_passes.mean())
 
