@@ -74,21 +74,13 @@ BLOCK_CASES = {
 }
 
 
-def forward_rows(cfg, tokens, block, tag):
-    """Oracle hidden states of the active block's rows after the last layer."""
-    P, BL = cfg["prompt_len"], cfg["block_len"]
-    h = np.stack([synth.weight_f64(cfg, -1, synth.EMBED, slice(int(t), int(t) + 1))[0] for t in tokens])
-    pos = np.arange(len(tokens))
-    t0 = time.time()
-    for l in range(cfg["n_layers"]):
-        h = O.layer_forward(cfg, synth.layer_weights_f64(cfg, l), h, pos)
-        print(f"{tag}: layer {l} done at {time.time() - t0:.0f} s", flush=True)
-    return h[P + block * BL: P + (block + 1) * BL]
-
-
 def run_blocks(preset: str) -> None:
-    """Cases already in the output file (same canvas seed) are kept, not recomputed."""
+    """Cases already in the output file (same canvas seed) are kept, not recomputed.
+    The missing cases go through the layers together: each layer's weights are
+    generated once and applied to every canvas (generating them is most of the
+    time), and the LM heads run once over all their active rows."""
     cfg = dict(configs.PRESETS[preset])
+    P, BL = cfg["prompt_len"], cfg["block_len"]
     path = os.path.join(HERE, f"fullsize_{preset}_blocks.json")
     done = {}
     if os.path.exists(path):
@@ -96,19 +88,27 @@ def run_blocks(preset: str) -> None:
             for c in json.load(f)["cases"]:
                 if c["canvas_seed"] == CANVAS_SEED:
                     done[(c["block"], c["frac_resolved"])] = c
-    cases = []
-    for block, frac in BLOCK_CASES[preset]:
-        if (block, frac) in done:
-            cases.append(done[(block, frac)])
-            continue
-        tokens, state = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, frac)
-        rows = forward_rows(cfg, tokens, block, f"{preset} block {block} frac {frac}")
-        cases.append({"block": block, "frac_resolved": frac, "canvas_seed": CANVAS_SEED,
-                      "heads": {"workload": head_eq1(cfg, rows),
-                                "gate_exercising": head_eq1(configs.gate_exercising(cfg), rows)}})
+    todo = [(b, fr) for b, fr in BLOCK_CASES[preset] if (b, fr) not in done]
+    if todo:
+        hs, pos = [], None
+        for block, frac in todo:
+            tokens, _ = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, frac)
+            hs.append(np.stack([synth.weight_f64(cfg, -1, synth.EMBED, slice(int(t), int(t) + 1))[0]
+                                for t in tokens]))
+            pos = np.arange(len(tokens))
+        t0 = time.time()
+        for l in range(cfg["n_layers"]):
+            lw = synth.layer_weights_f64(cfg, l)
+            hs = [O.layer_forward(cfg, lw, h, pos) for h in hs]
+            print(f"{preset}: {len(todo)} canvases, layer {l} done at {time.time() - t0:.0f} s", flush=True)
+        rows = np.concatenate([h[P + b * BL: P + (b + 1) * BL] for h, (b, _) in zip(hs, todo)])
+        heads = {"workload": head_eq1(cfg, rows), "gate_exercising": head_eq1(configs.gate_exercising(cfg), rows)}
+        for i, (block, frac) in enumerate(todo):
+            per = {name: {k: v[i * BL: (i + 1) * BL] for k, v in res.items()} for name, res in heads.items()}
+            done[(block, frac)] = {"block": block, "frac_resolved": frac, "canvas_seed": CANVAS_SEED, "heads": per}
     out = {"preset": preset, "sequence": 0,
            "source": "oracle/cora_oracle.py (layer_forward, lm_logits, top1, top2_margin), float64",
-           "cases": cases}
+           "cases": [done[c] for c in BLOCK_CASES[preset]]}
     with open(path, "w") as f:
         json.dump(out, f)
 
