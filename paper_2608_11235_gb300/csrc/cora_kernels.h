@@ -199,8 +199,9 @@ cudaError_t lm_head_prepare();
 cudaError_t attention_prepare();
 cudaError_t attention_tc_prepare();
 // tcgen05 attention for head_dim 128; tmQKV: bf16 [B*S, (Hq+2Hkv)*128], box 128 rows x 64 cols.
+// Persistent grid of min(items, num_sms) CTAs, items = ceil(q_len/128) * Hq * B.
 cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
-                                int q_len, int* err, cudaStream_t st);
+                                int q_len, int* err, int num_sms, cudaStream_t st);
 
 void launch_session_init(int32_t* tokens, const int32_t* prompt, uint8_t* state, int32_t* persist, int32_t* prev,
                          int32_t* ctrl, int32_t* status, int B, int P, int S, int G, int BL, int mask_id,

@@ -464,7 +464,7 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
     REC(CORA_KIND_GEMM_QKV);
     if (c.head_dim == 128) {
       CK(launch_attention_tc(cache ? s->tm_qkv_in_l[l] : s->tm_qkv_in, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads,
-                             lo, Ls, err, st));
+                             lo, Ls, err, m->num_sms, st));
     } else {
       launch_attention(qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, lo, Ls, st);
     }
@@ -1054,7 +1054,7 @@ extern "C" int cora_op_attention(const uint16_t* qkv, uint16_t* out, int32_t B, 
     const size_t cols = size_t(Hq + 2 * Hkv) * hd;
     if (!make_tmap_bf16_2d(&tq, qkv, size_t(B) * S, cols, cols * 2, 128, 64))
       return fail(CORA_ECUDA, "cora_op_attention: tensor map encoding failed");
-    CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, 0, S, dc->err, static_cast<cudaStream_t>(stream)));
+    CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, 0, S, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
   } else {
     launch_attention(qkv, out, B, S, Hq, Hkv, hd, 0, S, static_cast<cudaStream_t>(stream));
   }

@@ -157,9 +157,13 @@ def test_gemm_rope(B, S, H, Hkv, hd, theta):
 
 
 # --------------------------------------------------------------- attention
+# The last three head_dim-128 cases have more (sequence, head, query tile)
+# items than a GB300 has SMs, so persistent CTAs run several items each
+# (many key tiles per item; ragged; one key tile per item).
 @pytest.mark.parametrize("B,S,Hq,Hkv,hd", [(2, 96, 4, 4, 64), (1, 200, 8, 2, 128), (1, 512, 2, 2, 128),
                                           (2, 130, 4, 2, 128), (1, 1, 2, 2, 128), (2, 300, 4, 4, 128),
-                                          (3, 1, 2, 1, 64)])
+                                          (3, 1, 2, 1, 64), (4, 768, 28, 4, 128), (2, 1000, 16, 4, 128),
+                                          (40, 100, 8, 8, 128)])
 def test_attention(B, S, Hq, Hkv, hd):
     W = (Hq + 2 * Hkv) * hd
     qkv = bits(6, 10, (B * S, W), 1.0)
