@@ -206,6 +206,19 @@ def kernel_costs(cfg: dict):
     }
 
 
+def attn_kernel_name(cfg: dict) -> str:
+    """The attention kernel a dense pass of this workload launches: head_dim 64
+    runs the mma.sync kernel; head_dim 128 runs one CTA per (sequence, head,
+    128-query tile) item while the items fit on the SMs, else the persistent
+    kernel."""
+    if cfg["head_dim"] != 128:
+        return "attention_kernel"
+    import torch
+    items = -(-(cfg["prompt_len"] + cfg["gen_len"]) // 128) * cfg["n_heads"] * cfg["batch"]
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    return "attention_tc_kernel" if items <= sms else "attention_tc_persistent_kernel"
+
+
 def tiny_leg(reps: int = 5):
     """The tiny two-layer model at its own operating point (tau 0.9, K 2): GPU
     decode rate through cora_generate (device loop), passes per block, and the
@@ -440,7 +453,7 @@ def run_cora(args, cfg, ws, rank, local):
                          "peak": peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]),
                          "frac": round(head_gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]), 4),
                          "bytes_per_launch": costs["lm_head_top1_bytes"], "ms_per_launch": round(head_ms, 5)},
-        "attention": {"bound": "tensor", "kernel": "attention_tc_kernel" if cfg["head_dim"] == 128 else "attention_kernel",
+        "attention": {"bound": "tensor", "kernel": attn_kernel_name(cfg),
                       "achieved": round(costs["attention"] / (attn_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s",
                       "peak": peak_tf, "frac": round(costs["attention"] / (attn_ms * 1e-3) / 1e12 / peak_tf, 4),
                       "ms_per_launch": round(attn_ms, 5)},
