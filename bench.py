@@ -247,8 +247,8 @@ def tiny_leg(reps: int = 5):
     ora_s = _t.perf_counter() - t0
     return {"workload": cfg["name"], "tokens_per_s": round(G / gpu_s, 2), "passes": int(passes[0]),
             "passes_per_block": round(float(passes[0]) / (G // BL), 2), "timing": "host wall clock, cora_generate",
-            "oracle_generate_s": round(ora_s, 3), "oracle_passes": int(sum(tr.passes_per_block)),
-            "oracle_tokens_per_s": round(G / ora_s, 2)}
+            "cpu_baseline": {"kind": "oracle", "generate_s": round(ora_s, 3), "passes": int(sum(tr.passes_per_block)),
+                             "tokens_per_s": round(G / ora_s, 2), "sample": "the whole decode of the same prompt"}}
 
 
 def gate_isolation(peaks, reps: int = 5, with_oracle: bool = False):
