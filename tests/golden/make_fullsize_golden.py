@@ -117,34 +117,50 @@ CACHED_CASES = {"llada8b-shape-256+256": [(3, 0.5), (6, 0.75)]}  # (block, fract
 
 
 def run_cached(preset: str) -> None:
+    """Cases already in the output file (same canvas seed) are kept, not
+    recomputed; the missing ones go through the layers together, each layer's
+    weights generated once for all of them."""
     cfg = dict(configs.PRESETS[preset])
     P, BL = cfg["prompt_len"], cfg["block_len"]
     hkv, hd = cfg["n_kv_heads"], cfg["head_dim"]
-    cases = []
-    for block, frac in CACHED_CASES[preset]:
-        tok_a, _ = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, 0.0)   # the block's first pass
-        tok_b, _ = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, frac)  # a later pass of the block
-        lo = P + block * BL
-        assert np.array_equal(tok_a[:lo], tok_b[:lo])
+    path = os.path.join(HERE, f"fullsize_{preset}_cached.json")
+    done = {}
+    if os.path.exists(path):
+        with open(path) as f:
+            for c in json.load(f)["cases"]:
+                if c["canvas_seed"] == CANVAS_SEED:
+                    done[(c["block"], c["frac_resolved"])] = c
+    todo = [(b, fr) for b, fr in CACHED_CASES[preset] if (b, fr) not in done]
+    if todo:
         embed = lambda toks: np.stack([synth.weight_f64(cfg, -1, synth.EMBED, slice(int(t), int(t) + 1))[0]
                                        for t in toks])
-        ha, hb = embed(tok_a), embed(tok_b[lo:])
-        pos = np.arange(len(tok_a))
+        has, hbs, los, pos = [], [], [], None
+        for block, frac in todo:
+            tok_a, _ = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, 0.0)   # the block's first pass
+            tok_b, _ = synth.mid_decode_canvas(cfg, CANVAS_SEED, block, frac)  # a later pass of the block
+            lo = P + block * BL
+            assert np.array_equal(tok_a[:lo], tok_b[:lo])
+            has.append(embed(tok_a))
+            hbs.append(embed(tok_b[lo:]))
+            los.append(lo)
+            pos = np.arange(len(tok_a))
         empty = np.zeros((0, hkv, hd))
         t0 = time.time()
         for l in range(cfg["n_layers"]):
             lw = synth.layer_weights_f64(cfg, l)
-            ha, k, v = O.layer_forward_prefix(cfg, lw, ha, pos, empty, empty)
-            hb, _, _ = O.layer_forward_prefix(cfg, lw, hb, pos[lo:], k[:lo], v[:lo])
-            print(f"{preset} cached block {block} frac {frac}: layer {l} done at {time.time() - t0:.0f} s", flush=True)
-        rows = hb[:BL]
-        cases.append({"block": block, "frac_resolved": frac, "canvas_seed": CANVAS_SEED,
-                      "heads": {"workload": head_eq1(cfg, rows),
-                                "gate_exercising": head_eq1(configs.gate_exercising(cfg), rows)}})
+            for i, lo in enumerate(los):
+                has[i], k, v = O.layer_forward_prefix(cfg, lw, has[i], pos, empty, empty)
+                hbs[i], _, _ = O.layer_forward_prefix(cfg, lw, hbs[i], pos[lo:], k[:lo], v[:lo])
+            print(f"{preset} cached: {len(todo)} cases, layer {l} done at {time.time() - t0:.0f} s", flush=True)
+        rows = np.concatenate([hb[:BL] for hb in hbs])
+        heads = {"workload": head_eq1(cfg, rows), "gate_exercising": head_eq1(configs.gate_exercising(cfg), rows)}
+        for i, (block, frac) in enumerate(todo):
+            per = {name: {k: v[i * BL: (i + 1) * BL] for k, v in res.items()} for name, res in heads.items()}
+            done[(block, frac)] = {"block": block, "frac_resolved": frac, "canvas_seed": CANVAS_SEED, "heads": per}
     out = {"preset": preset, "sequence": 0,
            "source": "oracle/cora_oracle.py (layer_forward_prefix, lm_logits, top1, top2_margin), float64",
-           "cases": cases}
-    with open(os.path.join(HERE, f"fullsize_{preset}_cached.json"), "w") as f:
+           "cases": [done[c] for c in CACHED_CASES[preset]]}
+    with open(path, "w") as f:
         json.dump(out, f)
 
 
