@@ -210,3 +210,38 @@ def test_drift_threshold_value_printed_in_paper():
     # Table 1: the measured 1024/1024 GSM8K speedup is 92.7-99.5 % of the ideal 1/ratio.
     frac = float(fixture["gsm8k_1024_speedup"]) * float(fixture["gsm8k_1024_ratio"])
     assert 0.927 <= frac <= 0.995
+
+
+def test_top2_margin_closed_forms():
+    """p1 - p2 of softmax(l) (Eq. 1's distribution) against closed forms.
+
+    A margin taken on logits, or from the third-largest probability, or
+    without the softmax's normalisation, fails one of these."""
+    V = 50
+    assert abs(O.top2_margin(np.zeros((1, V)))[0]) < 1e-14                    # uniform: 0
+    l = np.zeros((1, V)); l[0, 3] = 4.0; l[0, 31] = 4.0                        # exact two-way top tie: 0
+    assert abs(O.top2_margin(l)[0]) < 1e-14
+    for g in (0.25, 2.0, 9.0):                                                 # one boosted id over V-1 zeros
+        l = np.zeros((1, V)); l[0, 11] = g
+        want = (math.exp(g) - 1.0) / (math.exp(g) + V - 1)
+        assert abs(O.top2_margin(l)[0] - want) < 1e-14
+    for a, b in ((3.0, 1.0), (6.0, 5.5), (0.7, 0.2)):                          # two boosted ids a > b
+        l = np.zeros((1, V)); l[0, 40] = a; l[0, 2] = b
+        want = (math.exp(a) - math.exp(b)) / (math.exp(a) + math.exp(b) + V - 2)
+        assert abs(O.top2_margin(l)[0] - want) < 1e-14
+    l = np.array([[-30.0, 0.0]])                                               # two-id vocabulary
+    assert abs(O.top2_margin(l)[0] - math.tanh(15.0)) < 1e-14
+
+
+def test_top2_margin_batched_rows_and_shift():
+    """[B, R, V] input gives the row-wise margins; a constant shift of a row changes nothing."""
+    rng = np.random.default_rng(12)
+    l = rng.normal(scale=3, size=(3, 5, 40))
+    m = O.top2_margin(l)
+    assert m.shape == (3, 5)
+    for b in range(3):
+        for r in range(5):
+            p = np.sort(softmax(l[b, r]))
+            assert abs(m[b, r] - (p[-1] - p[-2])) < 1e-14
+    assert np.allclose(O.top2_margin(l + 57.0), m, rtol=0, atol=1e-13)
+    assert np.all((m >= 0) & (m <= 1))
