@@ -95,36 +95,46 @@ typedef struct cora_model_config {
   float norm_eps;
 } cora_model_config;
 
-/* Weights, bf16 bit patterns in nn.Linear layout ([out_features,
- * in_features], row-major), "any" pointers.  Per-layer members point to host
- * arrays of n_layers tensor pointers.  Norm weights may be NULL (all ones).
+/* Weights in nn.Linear layout ([out_features, in_features], row-major),
+ * "any" pointers, every tensor of the element type `dtype` names:
+ *   CORA_DTYPE_BF16  bf16 bit patterns (uint16_t), copied as they are;
+ *   CORA_DTYPE_F32   IEEE float32, converted on the device to bf16 (round to
+ *                    nearest, ties to even), the precision the kernels
+ *                    compute in (the paper's backbones run in bf16, Sec. 4.1).
+ * Per-layer members point to host arrays of n_layers tensor pointers.  Norm
+ * weights may be NULL (all ones).
  *   embed    [vocab, d]           lm_head [vocab, d]        final_norm [d]
  *   wq [n_heads*hd, d]  wk, wv [n_kv_heads*hd, d]  wo [d, n_heads*hd]
  *   w_gate, w_up [ffn, d]         w_down [d, ffn]     attn_norm, ffn_norm [d]
  * The library copies them into its own device layout (fused QKV, gate/up
  * interleaved in 128-row groups, ffn padded to a multiple of 128 with zeros);
- * the caller may free its copies when cora_model_create returns. */
+ * float32 host tensors pass through a device staging buffer of at most
+ * 256 MiB.  The caller may free its copies when cora_model_create returns.
+ * A zero-initialised struct means bf16 (dtype 0). */
+#define CORA_DTYPE_BF16 0
+#define CORA_DTYPE_F32 1
 typedef struct cora_weights {
-  const uint16_t* embed;
-  const uint16_t* lm_head;
-  const uint16_t* final_norm;
-  const uint16_t* const* attn_norm;
-  const uint16_t* const* wq;
-  const uint16_t* const* wk;
-  const uint16_t* const* wv;
-  const uint16_t* const* wo;
-  const uint16_t* const* ffn_norm;
-  const uint16_t* const* w_gate;
-  const uint16_t* const* w_up;
-  const uint16_t* const* w_down;
+  const void* embed;
+  const void* lm_head;
+  const void* final_norm;
+  const void* const* attn_norm;
+  const void* const* wq;
+  const void* const* wk;
+  const void* const* wv;
+  const void* const* wo;
+  const void* const* ffn_norm;
+  const void* const* w_gate;
+  const void* const* w_up;
+  const void* const* w_down;
+  int32_t dtype; /* CORA_DTYPE_* */
 } cora_weights;
 
 typedef struct cora_model cora_model;
 typedef struct cora_session cora_session;
 
 /* Creates a device-resident model on the current device (synchronous).
- * Errors: CORA_EINVAL (config constraint, NULL tensor), CORA_ENOMEM,
- * CORA_ECUDA. */
+ * Errors: CORA_EINVAL (config constraint, NULL tensor, unknown dtype),
+ * CORA_ENOMEM, CORA_ECUDA. */
 CORA_API int cora_model_create(const cora_model_config* cfg, const cora_weights* w, cora_model** out);
 CORA_API int cora_model_destroy(cora_model* m);
 
@@ -188,14 +198,36 @@ CORA_API int cora_session_create_ex(cora_model* m, int32_t batch, const int32_t*
  * block/step/pass counter.  `prompt` is "any".  Synchronous. */
 CORA_API int cora_session_reset(cora_session* s, const int32_t* prompt);
 
-/* One executed denoising step for every unfinished sequence, at that
- * sequence's own (block, step): dense forward over the whole canvas, final
- * RMSNorm and LM head on the active block's rows only, Eq. 1 reduced on the
- * fly (logits never stored), then Eq. 2-4 and block termination.  Runs as one
- * CUDA graph on the session's stream and waits for it.
- *   all_done_out  host uint8: 1 once every sequence has finished all blocks
- * Errors: CORA_ESTATE (already finished), CORA_ETIMEOUT, CORA_ECUDA. */
-CORA_API int cora_denoise_step(cora_session* s, uint8_t* all_done_out);
+/* One executed denoising step (Sec. 3.1: step s of block b of the fixed
+ * horizon) for every unfinished sequence, at that sequence's own (block,
+ * step): dense forward over the whole canvas, final RMSNorm and LM head on the
+ * active block's rows only, Eq. 1 reduced on the fly (logits never stored),
+ * then the transfer rule, Eq. 2-4 and block termination.  Runs as one CUDA
+ * graph on the session's stream and waits for it.
+ *   block, step  the (block, step) the caller expects every unfinished
+ *                sequence to be at (0-based); -1 skips that check.  A
+ *                sequence at another block or step fails the call with
+ *                CORA_ESTATE before anything is launched (with B > 1 the
+ *                sequences may drift apart: pass -1 then).
+ *   conf_out     "any" float [B, block_len] or NULL (out): this step's c_i
+ *                (Eq. 1) of the rows of each sequence's active block
+ *   argmax_out   "any" int32 [B, block_len] or NULL (out): this step's x_hat_i
+ *                (Eq. 1), lowest id on ties
+ *                (CORA_PERSIST_CARRY sessions: both are [B, gen_len], one
+ *                entry per generation position)
+ *   done_out     "any" uint8 [B] or NULL (out): 1 when sequence b's block has
+ *                no unresolved position after this step (the block ended and
+ *                its remaining dense passes are skipped), or the sequence had
+ *                already finished; 0 otherwise
+ * Rows of a sequence that had finished before the step hold values computed
+ * and ignored.  Errors: CORA_ESTATE (already finished, or block/step differ),
+ * CORA_ETIMEOUT, CORA_ECUDA. */
+CORA_API int cora_denoise_step(cora_session* s, int32_t block, int32_t step, float* conf_out, int32_t* argmax_out,
+                               uint8_t* done_out);
+
+/* Host-side flag, no device work: *finished_out = 1 once every sequence of
+ * the session has finished all its blocks (as of the last completed call). */
+CORA_API int cora_session_finished(cora_session* s, uint8_t* finished_out);
 
 /* Runs cora_denoise_step until every sequence has finished (the decode loop
  * of Sec. 3, Fig. 2), as ONE graph launch: a conditional WHILE node around
@@ -326,14 +358,19 @@ CORA_API int cora_reduce_top1(const uint16_t* logits, int32_t rows, int32_t V, f
  * loops that must stay out of the allocator (cudaMalloc and cudaFree
  * synchronise the device).
  * Scratch is a fixed array compiled into the library (832 KiB: 65536 partial
- * states + 16384 counters), present on every GPU that loads the library until
- * the process exits.  Same arguments, layout and results as
+ * states + 16384 counters).  Same arguments, layout and results as
  * cora_reduce_top1; rows <= 16384, else CORA_EINVAL.
- * The first call on a device (with that device current) looks up the array's
- * device address; make that first call before any stream capture.  Calls
- * share the array, so calls that may overlap on the GPU (different streams
- * without ordering) race; serialise them.  Each call clears the counters it
- * uses with cudaMemsetAsync on `stream` before its kernel. */
+ * The array occupies device memory from the first use on a device of the
+ * library part that holds it (with CUDA's default lazy module loading: the
+ * first call of this function, or an earlier gate or Eq. 1 reduction call)
+ * until the process exits; later calls reserve nothing.  So make one call
+ * before a memory pool takes the whole device, and before any stream
+ * capture: that first call on a device (with that device current) also looks
+ * up the array's device address, which is then kept per device and looked up
+ * again only when the current context changes (e.g. after cudaDeviceReset).
+ * Calls share the array, so calls that may overlap on the GPU (different
+ * streams without ordering) race; serialise them.  Each call clears the
+ * counters it uses with cudaMemsetAsync on `stream` before its kernel. */
 CORA_API int cora_reduce_top1_noalloc(const uint16_t* logits, int32_t rows, int32_t V, float* conf, int32_t* argmax,
                                       void* stream);
 
@@ -375,6 +412,14 @@ CORA_API int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32_t
  * query head h reading KV head h / (Hq/Hkv). */
 CORA_API int cora_op_attention(const uint16_t* qkv, uint16_t* out, int32_t B, int32_t S, int32_t Hq, int32_t Hkv,
                       int32_t hd, void* stream);
+
+/* cora_op_attention for the queries q_start .. q_start + q_len - 1 of every
+ * sequence, against all S keys (the rows a prefix-cache pass recomputes;
+ * Sec. 5 composes the method with cache reuse): qkv as above, bf16
+ * [B*S, (Hq + 2*Hkv)*hd]; out bf16 [B*q_len, Hq*hd], q_len rows per
+ * sequence.  0 <= q_start, 1 <= q_len, q_start + q_len <= S. */
+CORA_API int cora_op_attention_rows(const uint16_t* qkv, uint16_t* out, int32_t B, int32_t S, int32_t Hq, int32_t Hkv,
+                                    int32_t hd, int32_t q_start, int32_t q_len, void* stream);
 
 /* RMSNorm rows: out bf16 [M, d] = x / sqrt(mean(x^2) + eps) * w, x fp32 [M, d],
  * w bf16 [d] (NULL = ones). */

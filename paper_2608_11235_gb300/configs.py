@@ -2,7 +2,9 @@
 
 Shapes follow the paper's backbones (LLaDA-8B and Dream-7B, Sec. 4.1) and its
 canvases (256/256 and 1024/1024 with block 32, Table 1); the tiny model is a
-two-layer stand-in small enough for the CPU oracle to decode end to end.
+two-layer stand-in small enough for the CPU oracle to decode end to end, with
+fp32 weights (the library rounds them to bf16 on the device; the oracle keeps
+the fp32 values), while the 8B-class shapes are bf16 models.
 Backbone constants the paper does not give (RoPE base, norm epsilon, untied
 head, unit norm weights) are fixed here once and handed to both the CUDA path
 and the oracle as plain numbers.
@@ -19,7 +21,7 @@ TINY = dict(
     name="tiny-2L-d256",
     n_layers=2, d_model=256, n_heads=4, n_kv_heads=4, head_dim=64, ffn=688,
     vocab=2048, mask_id=2047, rope_theta=10000.0, norm_eps=1e-5,
-    init_sigma=0.02, head_sigma=0.5, seed=0,
+    init_sigma=0.02, head_sigma=0.5, seed=0, weight_dtype="f32",
     batch=1, prompt_len=32, prompt_seed=100, gen_len=64, block_len=32, steps_per_block=32,
     tau=0.9, K=2,
 )

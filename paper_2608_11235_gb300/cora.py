@@ -27,7 +27,9 @@ EXPORTED = [
     "cora_op_gemm", "cora_op_attention", "cora_op_rmsnorm", "cora_op_lm_head_top1", "cora_synth_normal_bf16",
     "cora_device_error", "cora_session_profile_step", "cora_session_stream", "cora_reduce_top1_noalloc",
     "cora_session_create_ex", "cora_generate_ex", "cora_session_disagreement", "cora_check_wait_timeout",
+    "cora_session_finished", "cora_op_attention_rows",
 ]
+DTYPE_BF16, DTYPE_F32 = 0, 1
 SCHEDULE_FIXED, SCHEDULE_REMAINING = 0, 1
 PERSIST_BLOCK, PERSIST_CARRY = 0, 1
 CACHE_NONE, CACHE_PREFIX = 0, 1
@@ -61,7 +63,7 @@ PP = C.POINTER(C.c_void_p)
 class Weights(C.Structure):
     _fields_ = [("embed", C.c_void_p), ("lm_head", C.c_void_p), ("final_norm", C.c_void_p),
                 ("attn_norm", PP), ("wq", PP), ("wk", PP), ("wv", PP), ("wo", PP), ("ffn_norm", PP),
-                ("w_gate", PP), ("w_up", PP), ("w_down", PP)]
+                ("w_gate", PP), ("w_up", PP), ("w_down", PP), ("dtype", C.c_int32)]
 
 
 _lib = None
@@ -88,7 +90,8 @@ def lib():
             "cora_session_create": ([vp, i32, vp, i32, i32, i32, i32, f32, i32, C.POINTER(vp)], C.c_int),
             "cora_session_destroy": ([vp], C.c_int),
             "cora_session_reset": ([vp, vp], C.c_int),
-            "cora_denoise_step": ([vp, vp], C.c_int),
+            "cora_denoise_step": ([vp, i32, i32, vp, vp, vp], C.c_int),
+            "cora_session_finished": ([vp, vp], C.c_int),
             "cora_session_run": ([vp, vp, vp], C.c_int),
             "cora_session_read": ([vp] + [vp] * 9, C.c_int),
             "cora_session_write": ([vp] + [vp] * 5, C.c_int),
@@ -105,6 +108,7 @@ def lib():
             "cora_reduce_gate": ([vp, i32, i32, i32] + [vp] * 6 + [i32, f32, i32] + [vp] * 3 + [vp], C.c_int),
             "cora_op_gemm": ([vp, vp, vp, i32, i32, i32, i32, i32, vp, i32, i32, i32, vp], C.c_int),
             "cora_op_attention": ([vp, vp, i32, i32, i32, i32, i32, vp], C.c_int),
+            "cora_op_attention_rows": ([vp, vp, i32, i32, i32, i32, i32, i32, i32, vp], C.c_int),
             "cora_op_rmsnorm": ([vp, vp, vp, i32, i32, f32, vp], C.c_int),
             "cora_op_lm_head_top1": ([vp, vp, i32, i32, i32, vp, vp, vp], C.c_int),
             "cora_synth_normal_bf16": ([vp, i64, u64, i64, f32, vp], C.c_int),
@@ -147,10 +151,23 @@ def cora_version() -> int:
     return lib().cora_version()
 
 
+def _weight_dtype(t, default: int) -> int:
+    if not hasattr(t, "dtype"):          # raw addresses: the caller states the type
+        return default
+    name = str(t.dtype)
+    if "float32" in name:
+        return DTYPE_F32
+    if "int16" in name:
+        return DTYPE_BF16
+    raise TypeError(f"weights must be float32 or bf16 bit patterns (int16/uint16), got {name}")
+
+
 def cora_model_create(cfg: dict, tensors: dict) -> int:
-    """``tensors`` holds bf16-bit tensors (uint16/int16) in nn.Linear layout:
-    embed, lm_head, optional final_norm, and per-layer lists wq, wk, wv, wo,
-    w_gate, w_up, w_down, optional attn_norm / ffn_norm."""
+    """``tensors`` holds tensors in nn.Linear layout, all float32 or all bf16
+    bit patterns (uint16/int16): embed, lm_head, optional final_norm, and
+    per-layer lists wq, wk, wv, wo, w_gate, w_up, w_down, optional attn_norm /
+    ffn_norm.  The element type is passed to the library as cora_weights.dtype
+    (for raw integer addresses, from the optional ``dtype`` entry)."""
     c = ModelConfig(cfg["n_layers"], cfg["d_model"], cfg["n_heads"], cfg["n_kv_heads"], cfg["head_dim"],
                     cfg["ffn"], cfg["vocab"], cfg["mask_id"], cfg["rope_theta"], cfg["norm_eps"])
     L = cfg["n_layers"]
@@ -165,7 +182,7 @@ def cora_model_create(cfg: dict, tensors: dict) -> int:
 
     w = Weights(ptr(tensors["embed"]), ptr(tensors["lm_head"]), ptr(tensors.get("final_norm")),
                 arr("attn_norm"), arr("wq"), arr("wk"), arr("wv"), arr("wo"), arr("ffn_norm"),
-                arr("w_gate"), arr("w_up"), arr("w_down"))
+                arr("w_gate"), arr("w_up"), arr("w_down"), _weight_dtype(tensors["embed"], tensors.get("dtype", DTYPE_BF16)))
     out = C.c_void_p()
     _check("cora_model_create", lib().cora_model_create(C.byref(c), C.byref(w), C.byref(out)))
     return out.value
@@ -196,10 +213,21 @@ def cora_session_reset(session, prompt) -> None:
     _check("cora_session_reset", lib().cora_session_reset(session, ptr(prompt)))
 
 
-def cora_denoise_step(session) -> bool:
-    done = np.zeros(1, np.uint8)
-    _check("cora_denoise_step", lib().cora_denoise_step(session, ptr(done)))
-    return bool(done[0])
+def cora_denoise_step(session, block: int = -1, step: int = -1, conf_out=None, argmax_out=None,
+                      done_out=None) -> bool:
+    """One executed step (cora_denoise_step), then cora_session_finished:
+    returns True once every sequence has finished.  block/step = -1 skip the
+    check of the session's position; the outputs are optional [B, block_len]
+    float32 / int32 and [B] uint8 buffers (numpy or torch)."""
+    _check("cora_denoise_step", lib().cora_denoise_step(session, int(block), int(step), ptr(conf_out),
+                                                        ptr(argmax_out), ptr(done_out)))
+    return cora_session_finished(session)
+
+
+def cora_session_finished(session) -> bool:
+    out = np.zeros(1, np.uint8)
+    _check("cora_session_finished", lib().cora_session_finished(session, ptr(out)))
+    return bool(out[0])
 
 
 def cora_session_run(session) -> tuple:
@@ -310,6 +338,11 @@ def cora_op_gemm(A, B, Cm, M, N, K, ldc, epilogue, rope=None, seq=0, head_dim=0,
 
 def cora_op_attention(qkv, out, B, S, Hq, Hkv, hd, stream=None) -> None:
     _check("cora_op_attention", lib().cora_op_attention(ptr(qkv), ptr(out), B, S, Hq, Hkv, hd, _stream(stream)))
+
+
+def cora_op_attention_rows(qkv, out, B, S, Hq, Hkv, hd, q_start, q_len, stream=None) -> None:
+    _check("cora_op_attention_rows", lib().cora_op_attention_rows(ptr(qkv), ptr(out), B, S, Hq, Hkv, hd, q_start,
+                                                                  q_len, _stream(stream)))
 
 
 def cora_op_rmsnorm(x, w, out, M, d, eps, stream=None) -> None:

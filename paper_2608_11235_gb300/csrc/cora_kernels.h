@@ -53,6 +53,7 @@ struct SessionGateArgs {
   uint8_t* unmask;        // [B][BL]
   uint8_t* accept;        // [B][BL]
   uint8_t* all_done;      // [1]
+  uint8_t* blk_done;      // [B]: 1 when the sequence's block has no unresolved position after the step
   int* err;
   int B, S, P, G, BL, T;
   float tau;
@@ -70,6 +71,10 @@ struct SessionGateArgs {
   int lockstep;
 };
 
+// dst (bf16 bits, row stride dst_ld elements) = round-to-nearest-even of the
+// fp32 block src [rows, cols] (row stride src_ld elements); device pointers.
+void launch_f32_to_bf16_2d(const float* src, int64_t src_ld, uint16_t* dst, int64_t dst_ld, int64_t rows,
+                           int64_t cols, cudaStream_t st);
 void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_t start, float scale,
                               cudaStream_t st);
 void launch_embed(const int32_t* tokens, const uint16_t* embed, float* h, int M, int d, int S_tok, int lo,

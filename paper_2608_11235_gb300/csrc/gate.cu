@@ -3,6 +3,8 @@
 #include <float.h>
 #include <limits.h>
 
+#include <cudaTypedefs.h>
+
 #include <mutex>
 
 #include "cora_device.cuh"
@@ -284,8 +286,12 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
   __syncthreads();
   for (int b = threadIdx.x >> 5; b < a.B; b += nw) {
     int32_t* ctrl = a.ctrl + b * 4;
-    if (ctrl[3]) continue;                   // finished: nothing to do (warp-uniform)
-    if (a.lockstep && ctrl[1] < 0) continue;  // block ended, waiting for the other sequences
+    if (ctrl[3] || (a.lockstep && ctrl[1] < 0)) {
+      // finished, or (prefix cache) block ended and waiting for the other
+      // sequences: nothing to do (warp-uniform); no unresolved position left
+      if (lane == 0) a.blk_done[b] = 1;
+      continue;
+    }
     const int blk = ctrl[0], step = ctrl[1];
     if (carry) {
       // Carry-over persistence: Eq. 2 for every unresolved generation
@@ -344,6 +350,7 @@ __global__ void session_gate_kernel(SessionGateArgs a) {
     }
     __syncwarp();
     if (lane == 0) {
+      a.blk_done[b] = blk_done ? 1 : 0;
       ctrl[2] += 1;  // executed passes of this sequence
       if (blk_done && a.lockstep && !eos_stop && blk + 1 < n_blocks) {
         ctrl[1] = -1;  // wait: the sequences move to the next block together
@@ -483,9 +490,18 @@ void launch_session_gate(const SessionGateArgs& a, cudaStream_t st) {
 // reduction: an application whose memory pool already owns the whole device
 // (a cudaMalloc would fail or force it to give memory back), or a
 // latency-critical loop that must not enter the allocator (cudaMalloc and
-// cudaFree synchronise the device).  cora_reduce_top1_noalloc serves them with scratch that exists as
-// soon as the library is loaded: the array below, reserved on every GPU that
-// loads the library and kept until the process exits.
+// cudaFree synchronise the device).  cora_reduce_top1_noalloc serves them with
+// the fixed array below instead of allocated scratch.
+//
+// When the array occupies device memory: this file is its own CUDA module,
+// and with lazy module loading (the default since CUDA 12.2) a module is put
+// on a device the first time one of its kernels or symbols is used there.  So
+// the array is reserved on a device at the first use of this file's code on
+// that device: the first cora_reduce_top1_noalloc call, or earlier any other
+// call whose kernels live here (the gate and Eq. 1 reductions).  From then on
+// it stays until the process exits (or its context is destroyed), and calls
+// reserve nothing more.  A caller whose memory pool will take the whole device
+// therefore makes one call before the pool does.
 // ----------------------------------------------------------------------------
 #define CORA_NOALLOC_MAX_PARTIALS 65536  // (chunk, row) partial states: 768 KiB
 #define CORA_NOALLOC_MAX_ROWS 16384      // completion counters: 64 KiB
@@ -499,8 +515,33 @@ static __device__ __align__(256) NoAllocScratch g_noalloc_scratch;
 
 namespace {
 std::mutex g_noalloc_mu;
-NoAllocScratch* g_noalloc_dev[64];  // device address of the array, per device
+// Device address of the array per device, valid for the context it was looked
+// up in: a context destroyed by cudaDeviceReset (or a module reloaded in a new
+// context) invalidates it, so it is looked up again when the current
+// context's unique id differs.
+NoAllocScratch* g_noalloc_dev[64];
+unsigned long long g_noalloc_ctx[64];
 int g_noalloc_sms[64];
+PFN_cuCtxGetCurrent_v4000 g_ctx_current = nullptr;
+PFN_cuCtxGetId_v12000 g_ctx_id = nullptr;
+
+// Unique id of the calling thread's current context; false if none is
+// current yet or it cannot be read.
+bool current_context_id(unsigned long long* id) {
+  if (!g_ctx_current || !g_ctx_id) {
+    cudaDriverEntryPointQueryResult q1, q2;
+    void *f1 = nullptr, *f2 = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f1, 4000, cudaEnableDefault, &q1) != cudaSuccess ||
+        cudaGetDriverEntryPointByVersion("cuCtxGetId", &f2, 12000, cudaEnableDefault, &q2) != cudaSuccess ||
+        q1 != cudaDriverEntryPointSuccess || q2 != cudaDriverEntryPointSuccess || !f1 || !f2)
+      return false;
+    g_ctx_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(f1);
+    g_ctx_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(f2);
+  }
+  CUcontext ctx = nullptr;
+  if (g_ctx_current(&ctx) != CUDA_SUCCESS || !ctx) return false;
+  return g_ctx_id(ctx, id) == CUDA_SUCCESS;
+}
 }  // namespace
 
 extern "C" int cora_reduce_top1_noalloc(const uint16_t* logits, int32_t rows, int32_t V, float* conf, int32_t* argmax,
@@ -517,16 +558,25 @@ extern "C" int cora_reduce_top1_noalloc(const uint16_t* logits, int32_t rows, in
   NoAllocScratch* scratch = nullptr;
   int num_sms = 0;
   {
-    // First call on a device: look up where the array lives on that device
-    // (the array's name is only a host-side handle) and the SM count.
+    // First call on a device (or in a new context on it): look up where the
+    // array lives there (the array's name is only a host-side handle) and the
+    // SM count.
     std::lock_guard<std::mutex> lk(g_noalloc_mu);
-    if (!g_noalloc_dev[dev]) {
+    unsigned long long ctx_id = 0;
+    const bool have_ctx = current_context_id(&ctx_id);
+    if (!have_ctx || !g_noalloc_dev[dev] || g_noalloc_ctx[dev] != ctx_id) {
+      g_noalloc_dev[dev] = nullptr;
       void* p = nullptr;
+      // (the runtime makes the device's primary context current here if no
+      // context is current yet)
       if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
         return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: cudaGetSymbolAddress failed");
+      if (!current_context_id(&ctx_id))
+        return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: cannot read the current context");
       if (cudaDeviceGetAttribute(&g_noalloc_sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return cora_set_error(CORA_ECUDA, "cora_reduce_top1_noalloc: cannot read the SM count");
       g_noalloc_dev[dev] = static_cast<NoAllocScratch*>(p);
+      g_noalloc_ctx[dev] = ctx_id;
     }
     scratch = g_noalloc_dev[dev];
     num_sms = g_noalloc_sms[dev];

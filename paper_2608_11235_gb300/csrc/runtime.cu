@@ -52,7 +52,7 @@ int cora_set_error(int code, const char* msg) {
   } while (0)
 
 extern "C" const char* cora_last_error(void) { return g_last_error.c_str(); }
-extern "C" int cora_version(void) { return 100; }
+extern "C" int cora_version(void) { return 200; }
 
 // --------------------------------------------------------- device context
 namespace {
@@ -212,9 +212,60 @@ static void model_free(cora_model* m) {
   m->allocs.clear();
 }
 
-static int copy_rows(uint16_t* dst, const uint16_t* src, size_t rows, size_t cols) {
-  CK(cudaMemcpy(dst, src, rows * cols * 2, cudaMemcpyDefault));
+// Weight upload: [rows, cols] elements of `dtype` at src (row stride src_ld
+// elements, "any" pointer) into bf16 dst (row stride dst_ld).  bf16 is copied
+// as it is; fp32 is rounded to bf16 on the device, read in place when the
+// caller's tensor is device-accessible, else through the staging buffer.
+struct WeightUpload {
+  int dtype = CORA_DTYPE_BF16;
+  float* stage = nullptr;  // device staging buffer for fp32 host tensors
+  size_t stage_elems = 0;
+  ~WeightUpload() {
+    if (stage) cudaFree(stage);
+  }
+};
+constexpr size_t kStageBytes = size_t(256) << 20;
+
+static size_t dtype_bytes(int dtype) { return dtype == CORA_DTYPE_F32 ? 4 : 2; }
+
+static const void* elem_offset(const void* p, size_t elems, int dtype) {
+  return static_cast<const char*>(p) + elems * dtype_bytes(dtype);
+}
+
+static int put_rows(WeightUpload& up, uint16_t* dst, size_t dst_ld, const void* src, size_t src_ld, size_t rows,
+                    size_t cols) {
+  if (up.dtype == CORA_DTYPE_BF16) {
+    CK(cudaMemcpy2D(dst, dst_ld * 2, src, src_ld * 2, cols * 2, rows, cudaMemcpyDefault));
+    return CORA_OK;
+  }
+  cudaPointerAttributes at{};
+  CK(cudaPointerGetAttributes(&at, src));
+  if (at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged) {
+    launch_f32_to_bf16_2d(static_cast<const float*>(src), int64_t(src_ld), dst, int64_t(dst_ld), int64_t(rows),
+                          int64_t(cols), nullptr);
+    CK(cudaGetLastError());
+    CK(cudaDeviceSynchronize());
+    return CORA_OK;
+  }
+  if (!up.stage) {
+    up.stage_elems = kStageBytes / 4;
+    CK(cudaMalloc(&up.stage, up.stage_elems * 4));
+  }
+  const size_t rows_per_chunk = std::max<size_t>(1, up.stage_elems / cols);
+  for (size_t r0 = 0; r0 < rows; r0 += rows_per_chunk) {
+    const size_t n = std::min(rows_per_chunk, rows - r0);
+    CK(cudaMemcpy2D(up.stage, cols * 4, elem_offset(src, r0 * src_ld, CORA_DTYPE_F32), src_ld * 4, cols * 4, n,
+                    cudaMemcpyHostToDevice));
+    launch_f32_to_bf16_2d(up.stage, int64_t(cols), dst + r0 * dst_ld, int64_t(dst_ld), int64_t(n), int64_t(cols),
+                          nullptr);
+    CK(cudaGetLastError());
+    CK(cudaDeviceSynchronize());  // the staging buffer is reused by the next chunk
+  }
   return CORA_OK;
+}
+
+static int copy_rows(WeightUpload& up, uint16_t* dst, const void* src, size_t rows, size_t cols) {
+  return put_rows(up, dst, cols, src, cols, rows, cols);
 }
 
 extern "C" int cora_model_destroy(cora_model* m);
@@ -231,6 +282,8 @@ extern "C" int cora_model_create(const cora_model_config* cfg, const cora_weight
           "(n_heads + 2 n_kv_heads) * head_dim must be a multiple of 128");
   REQUIRE(c.ffn >= 1 && c.vocab >= 2 && c.mask_id >= 0 && c.mask_id < c.vocab, "bad ffn/vocab/mask_id");
   REQUIRE(c.norm_eps >= 0.f && c.rope_theta > 0.f, "bad norm_eps/rope_theta");
+  REQUIRE(w->dtype == CORA_DTYPE_BF16 || w->dtype == CORA_DTYPE_F32, "cora_model_create: unknown weight dtype %d",
+          w->dtype);
   REQUIRE(w->embed && w->lm_head && w->wq && w->wk && w->wv && w->wo && w->w_gate && w->w_up && w->w_down,
           "cora_model_create: NULL weight");
   for (int l = 0; l < c.n_layers; ++l)
@@ -259,41 +312,44 @@ extern "C" int cora_model_create(const cora_model_config* cfg, const cora_weight
     }                     \
   } while (0)
 
+  WeightUpload up;
+  up.dtype = w->dtype;
+  const int dt = w->dtype;
   MK(model_alloc(m, size_t(c.vocab) * d * 2, &m->embed));
-  MK(copy_rows(m->embed, w->embed, c.vocab, d));
+  MK(copy_rows(up, m->embed, w->embed, c.vocab, d));
   MK(model_alloc(m, size_t(c.vocab) * d * 2, &m->head));
-  MK(copy_rows(m->head, w->lm_head, c.vocab, d));
+  MK(copy_rows(up, m->head, w->lm_head, c.vocab, d));
   if (w->final_norm) {
     MK(model_alloc(m, d * 2, &m->final_norm));
-    MK(copy_rows(m->final_norm, w->final_norm, 1, d));
+    MK(copy_rows(up, m->final_norm, w->final_norm, 1, d));
   }
   for (int l = 0; l < c.n_layers; ++l) {
     uint16_t *an = nullptr, *fn = nullptr, *qkv, *wo, *gu, *dn;
     if (w->attn_norm && w->attn_norm[l]) {
       MK(model_alloc(m, d * 2, &an));
-      MK(copy_rows(an, w->attn_norm[l], 1, d));
+      MK(copy_rows(up, an, w->attn_norm[l], 1, d));
     }
     if (w->ffn_norm && w->ffn_norm[l]) {
       MK(model_alloc(m, d * 2, &fn));
-      MK(copy_rows(fn, w->ffn_norm[l], 1, d));
+      MK(copy_rows(up, fn, w->ffn_norm[l], 1, d));
     }
     MK(model_alloc(m, size_t(m->n_qkv) * d * 2, &qkv));
-    MK(copy_rows(qkv, w->wq[l], hq, d));
-    MK(copy_rows(qkv + hq * d, w->wk[l], hkv, d));
-    MK(copy_rows(qkv + (hq + hkv) * d, w->wv[l], hkv, d));
+    MK(copy_rows(up, qkv, w->wq[l], hq, d));
+    MK(copy_rows(up, qkv + hq * d, w->wk[l], hkv, d));
+    MK(copy_rows(up, qkv + (hq + hkv) * d, w->wv[l], hkv, d));
     MK(model_alloc(m, d * hq * 2, &wo));
-    MK(copy_rows(wo, w->wo[l], d, hq));
+    MK(copy_rows(up, wo, w->wo[l], d, hq));
     // gate/up interleaved in groups of 128 rows: [gate 128 | up 128] per group.
     MK(model_alloc(m, 2 * FP * d * 2, &gu));
     if (FP != F) CK(cudaMemset(gu, 0, 2 * FP * d * 2));
     for (size_t g0 = 0; g0 < F; g0 += 128) {
       const size_t n = (F - g0) < 128 ? (F - g0) : 128;
-      MK(copy_rows(gu + (2 * g0) * d, w->w_gate[l] + g0 * d, n, d));
-      MK(copy_rows(gu + (2 * g0 + 128) * d, w->w_up[l] + g0 * d, n, d));
+      MK(copy_rows(up, gu + (2 * g0) * d, elem_offset(w->w_gate[l], g0 * d, dt), n, d));
+      MK(copy_rows(up, gu + (2 * g0 + 128) * d, elem_offset(w->w_up[l], g0 * d, dt), n, d));
     }
     MK(model_alloc(m, d * FP * 2, &dn));
     if (FP != F) CK(cudaMemset(dn, 0, d * FP * 2));
-    CK(cudaMemcpy2D(dn, FP * 2, w->w_down[l], F * 2, F * 2, d, cudaMemcpyDefault));
+    MK(put_rows(up, dn, FP, w->w_down[l], F, d, F));
     m->attn_norm.push_back(an);
     m->ffn_norm.push_back(fn);
     m->wqkv.push_back(qkv);
@@ -354,6 +410,7 @@ struct cora_session {
   int32_t* argmax = nullptr;   // [B, BL]
   uint8_t* unmask = nullptr;   // [B, BL]
   uint8_t* accept = nullptr;   // [B, BL]
+  uint8_t* blk_done = nullptr; // [B] block had no unresolved position after the last step
   int32_t* status = nullptr;   // device {all_done (byte 0), error word}
   int32_t* status_h = nullptr; // pinned host copy
   long long* diag = nullptr;   // [B][3] disagreement counts
@@ -498,7 +555,7 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
   }
   SessionGateArgs ga{s->parts, s->n_parts, s->ctrl,  s->tokens, s->state,  s->persist, s->prev,
                      s->conf,  s->argmax,  s->unmask, s->accept, reinterpret_cast<uint8_t*>(s->status),
-                     err,      s->B,       s->S,      s->P,      s->G,       s->BL,      s->T,
+                     s->blk_done, err,      s->B,       s->S,      s->P,      s->G,       s->BL,      s->T,
                      s->tau,   s->K,       s->opt.schedule, s->opt.eos_id, s->rows_per_seq, s->chunk_rows,
                      cache ? 1 : 0};
   launch_session_gate(ga, st);
@@ -656,6 +713,7 @@ extern "C" int cora_session_create_ex(cora_model* m, int32_t batch, const int32_
   SK(sess_alloc(s, size_t(s->Re), &s->argmax));
   SK(sess_alloc(s, size_t(s->R), &s->unmask));
   SK(sess_alloc(s, size_t(s->R), &s->accept));
+  SK(sess_alloc(s, size_t(batch), &s->blk_done));
   SK(sess_alloc(s, 4, &s->status));
   SK(sess_alloc(s, size_t(batch) * 3, &s->diag));
   SK(sess_alloc(s, gemm_workspace_bytes(m->num_sms) / sizeof(float), &s->gemm_ws.partial));
@@ -761,8 +819,9 @@ extern "C" int cora_model_destroy(cora_model* m) {
   return CORA_OK;
 }
 
-extern "C" int cora_denoise_step(cora_session* s, uint8_t* all_done_out) {
-  REQUIRE(s, "cora_denoise_step: NULL session");
+// One graph launch of the step at every unfinished sequence's own (block,
+// step); waits for it and reads the status word.
+static int step_once(cora_session* s, uint8_t* all_done_out) {
   if (s->finished) return fail(CORA_ESTATE, "every sequence has finished; reset the session");
   cudaGraphExec_t g = s->graph;
   if (!s->cgraph.empty() && !(s->next_info & 1)) {
@@ -782,6 +841,37 @@ extern "C" int cora_denoise_step(cora_session* s, uint8_t* all_done_out) {
   return CORA_OK;
 }
 
+extern "C" int cora_denoise_step(cora_session* s, int32_t block, int32_t step, float* conf_out, int32_t* argmax_out,
+                                 uint8_t* done_out) {
+  REQUIRE(s, "cora_denoise_step: NULL session");
+  REQUIRE(block >= -1 && step >= -1, "cora_denoise_step: block and step must be >= 0, or -1 for no check");
+  if (s->finished) return fail(CORA_ESTATE, "every sequence has finished; reset the session");
+  if (block >= 0 || step >= 0) {
+    std::vector<int32_t> ctrl(size_t(s->B) * 4);
+    CK(cudaStreamSynchronize(s->stream));
+    CK(cudaMemcpy(ctrl.data(), s->ctrl, ctrl.size() * 4, cudaMemcpyDeviceToHost));
+    for (int b = 0; b < s->B; ++b) {
+      const int32_t* c = &ctrl[size_t(b) * 4];
+      if (c[3] || c[1] < 0) continue;  // finished, or waiting for the batch's next block (prefix cache)
+      if ((block >= 0 && c[0] != block) || (step >= 0 && c[1] != step))
+        return fail(CORA_ESTATE, "cora_denoise_step: sequence %d is at block %d step %d, not block %d step %d", b,
+                    c[0], c[1], block, step);
+    }
+  }
+  const int rc = step_once(s, nullptr);
+  if (rc) return rc;
+  if (conf_out) CK(cudaMemcpy(conf_out, s->conf, size_t(s->Re) * 4, cudaMemcpyDefault));
+  if (argmax_out) CK(cudaMemcpy(argmax_out, s->argmax, size_t(s->Re) * 4, cudaMemcpyDefault));
+  if (done_out) CK(cudaMemcpy(done_out, s->blk_done, size_t(s->B), cudaMemcpyDefault));
+  return CORA_OK;
+}
+
+extern "C" int cora_session_finished(cora_session* s, uint8_t* finished_out) {
+  REQUIRE(s && finished_out, "cora_session_finished: NULL argument");
+  *finished_out = s->finished ? 1 : 0;
+  return CORA_OK;
+}
+
 extern "C" int cora_session_run(cora_session* s, int32_t* steps_out, uint8_t* on_device_out) {
   REQUIRE(s, "cora_session_run: NULL session");
   if (s->finished) return fail(CORA_ESTATE, "every sequence has finished; reset the session");
@@ -798,7 +888,7 @@ extern "C" int cora_session_run(cora_session* s, int32_t* steps_out, uint8_t* on
   } else {
     uint8_t done = 0;
     for (int32_t i = 0; i < s->max_iters && !done; ++i, ++steps) {
-      const int rc = cora_denoise_step(s, &done);
+      const int rc = step_once(s, &done);
       if (rc) return rc;
     }
   }
@@ -1039,11 +1129,20 @@ extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32
   return CORA_OK;
 }
 
+extern "C" int cora_op_attention_rows(const uint16_t* qkv, uint16_t* out, int32_t B, int32_t S, int32_t Hq,
+                                      int32_t Hkv, int32_t hd, int32_t q_start, int32_t q_len, void* stream);
+
 extern "C" int cora_op_attention(const uint16_t* qkv, uint16_t* out, int32_t B, int32_t S, int32_t Hq, int32_t Hkv,
                                  int32_t hd, void* stream) {
+  return cora_op_attention_rows(qkv, out, B, S, Hq, Hkv, hd, 0, S, stream);
+}
+
+extern "C" int cora_op_attention_rows(const uint16_t* qkv, uint16_t* out, int32_t B, int32_t S, int32_t Hq,
+                                      int32_t Hkv, int32_t hd, int32_t q_start, int32_t q_len, void* stream) {
   REQUIRE(qkv && out, "cora_op_attention: NULL pointer");
   REQUIRE(B >= 1 && S >= 1 && Hq >= 1 && Hkv >= 1 && Hq % Hkv == 0 && (hd == 64 || hd == 128),
           "cora_op_attention: bad shape");
+  REQUIRE(q_start >= 0 && q_len >= 1 && int64_t(q_start) + q_len <= S, "cora_op_attention: bad query range");
   REQUIRE(aligned16(qkv) && aligned16(out), "cora_op_attention: pointers must be 16-byte aligned");
   int rc = kernels_prepare();
   if (rc) return rc;
@@ -1054,9 +1153,10 @@ extern "C" int cora_op_attention(const uint16_t* qkv, uint16_t* out, int32_t B, 
     const size_t cols = size_t(Hq + 2 * Hkv) * hd;
     if (!make_tmap_bf16_2d(&tq, qkv, size_t(B) * S, cols, cols * 2, 128, 64))
       return fail(CORA_ECUDA, "cora_op_attention: tensor map encoding failed");
-    CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, 0, S, dc->err, dc->num_sms, static_cast<cudaStream_t>(stream)));
+    CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, q_start, q_len, dc->err, dc->num_sms,
+                           static_cast<cudaStream_t>(stream)));
   } else {
-    launch_attention(qkv, out, B, S, Hq, Hkv, hd, 0, S, static_cast<cudaStream_t>(stream));
+    launch_attention(qkv, out, B, S, Hq, Hkv, hd, q_start, q_len, static_cast<cudaStream_t>(stream));
   }
   CK(cudaGetLastError());
   return CORA_OK;

@@ -27,6 +27,18 @@ __global__ void synth_normal_bf16_kernel(uint16_t* __restrict__ out, int64_t cou
   }
 }
 
+// dst[r, c] = bf16(src[r, c]) for a [rows, cols] fp32 block (row strides in
+// elements), round to nearest even: the fp32 weight input of the model.
+__global__ void f32_to_bf16_2d_kernel(const float* __restrict__ src, int64_t src_ld, uint16_t* __restrict__ dst,
+                                      int64_t dst_ld, int64_t rows, int64_t cols) {
+  const int64_t n = rows * cols;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n; i += stride) {
+    const int64_t r = i / cols, c = i - r * cols;
+    dst[r * dst_ld + c] = __bfloat16_as_ushort(__float2bfloat16_rn(src[r * src_ld + c]));
+  }
+}
+
 // h[r, :] = float(embed[tokens[r], :]); one warp per row, 16-byte loads.
 // Row r of h takes token r of the canvas, or, with rows_per_seq > 0 (packed
 // rows of a prefix-cache pass), token lo + r % rows_per_seq of sequence
@@ -204,6 +216,15 @@ void launch_session_init(int32_t* tokens, const int32_t* prompt, uint8_t* state,
   if (blocks > 4096) blocks = 4096 > need ? 4096 : need;
   session_init_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(tokens, prompt, state, persist, prev, ctrl, status, B,
                                                                  P, S, G, BL, mask_id);
+}
+
+void launch_f32_to_bf16_2d(const float* src, int64_t src_ld, uint16_t* dst, int64_t dst_ld, int64_t rows,
+                           int64_t cols, cudaStream_t st) {
+  const int64_t n = rows * cols;
+  int64_t blocks = (n + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  if (blocks < 1) blocks = 1;
+  f32_to_bf16_2d_kernel<<<static_cast<int>(blocks), 256, 0, st>>>(src, src_ld, dst, dst_ld, rows, cols);
 }
 
 void launch_synth_normal_bf16(uint16_t* out, int64_t count, uint64_t key, int64_t start, float scale,

@@ -19,13 +19,16 @@ second implementation of the same generator (``cora_synth_normal_bf16``) so the
 8B-parameter weights can be written straight into device memory, and a test
 checks the two bit for bit.
 
-Weights are bf16-representable by construction.  An approximate N(0, sigma)
-sample is the Irwin-Hall sum of the four 16-bit fields of one 64-bit output:
-``X = 2*(u0+u1+u2+u3) - 4*65535`` (an odd integer, |X| <= 262140, exact in
-fp32), scaled by the fp32 constant ``sigma / SD_X`` with one IEEE fp32
-multiply and rounded to bf16 (round to nearest even).  Integer fields, one
-fp32 multiply and an integer rounding step give the same bits on any IEEE
-machine.
+An approximate N(0, sigma) sample is the Irwin-Hall sum of the four 16-bit
+fields of one 64-bit output: ``X = 2*(u0+u1+u2+u3) - 4*65535`` (an odd
+integer, |X| <= 262140, exact in fp32), scaled by the fp32 constant
+``sigma / SD_X`` with one IEEE fp32 multiply.  A workload whose weights are
+bf16 (``weight_dtype`` "bf16", the default) rounds that product to bf16
+(round to nearest even), so both sides see identical values; a workload with
+fp32 weights (``weight_dtype`` "f32", the tiny model) keeps the fp32 product,
+which in general is not bf16-representable: the oracle computes with it and
+the library rounds it to bf16 on the device.  Integer fields, one fp32
+multiply and an integer rounding step give the same bits on any IEEE machine.
 """
 
 from __future__ import annotations
@@ -93,13 +96,18 @@ def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
     return (np.asarray(b, dtype=np.uint16).astype(np.uint32) << np.uint32(16)).view(np.float32)
 
 
-def normal_bf16_bits(key: int, start: int, count: int, sigma: float) -> np.ndarray:
-    """Approximate N(0, sigma) samples as bf16 bit patterns (see module doc)."""
+def normal_f32(key: int, start: int, count: int, sigma: float) -> np.ndarray:
+    """Approximate N(0, sigma) samples in fp32: X times the fp32 scale (see module doc)."""
     b = bits64(key, start, count)
     m = np.uint64(0xFFFF)
     s = (b & m) + ((b >> np.uint64(16)) & m) + ((b >> np.uint64(32)) & m) + (b >> np.uint64(48))
     x = (2 * s.astype(np.int64) - 4 * 65535).astype(np.float32)
-    return f32_to_bf16_bits(x * normal_scale_f32(sigma))
+    return x * normal_scale_f32(sigma)
+
+
+def normal_bf16_bits(key: int, start: int, count: int, sigma: float) -> np.ndarray:
+    """Approximate N(0, sigma) samples as bf16 bit patterns (see module doc)."""
+    return f32_to_bf16_bits(normal_f32(key, start, count, sigma))
 
 
 def uniform_int(key: int, start: int, count: int, n: int) -> np.ndarray:
@@ -151,7 +159,23 @@ def weight_bf16_bits(cfg: dict, layer: int, kind: int, rows: slice | None = None
     return out.reshape(r1 - r0, shp[1])
 
 
+def weight_f32(cfg: dict, layer: int, kind: int, rows: slice | None = None) -> np.ndarray:
+    """fp32 values of one weight tensor of an fp32-weight workload (not rounded to bf16)."""
+    shp = weight_shapes(cfg)[kind]
+    r0, r1 = (0, shp[0]) if rows is None else (rows.start or 0, rows.stop)
+    key = stream_key(cfg["seed"], tensor_stream(layer, kind))
+    return normal_f32(key, r0 * shp[1], (r1 - r0) * shp[1], weight_sigma(cfg, kind)).reshape(r1 - r0, shp[1])
+
+
+def is_f32_weights(cfg: dict) -> bool:
+    return cfg.get("weight_dtype", "bf16") == "f32"
+
+
 def weight_f64(cfg: dict, layer: int, kind: int, rows: slice | None = None) -> np.ndarray:
+    """The workload's weight values widened to float64: the fp32 originals of an
+    fp32-weight workload, else the bf16 values."""
+    if is_f32_weights(cfg):
+        return weight_f32(cfg, layer, kind, rows).astype(np.float64)
     return bf16_bits_to_f32(weight_bf16_bits(cfg, layer, kind, rows)).astype(np.float64)
 
 

@@ -32,7 +32,7 @@ def test_every_declared_symbol_is_exported(L):
 
 
 def test_version(L):
-    assert cora.cora_version() == 100
+    assert cora.cora_version() == 200
 
 
 def test_invalid_arguments_rejected_before_launch(L):
@@ -87,3 +87,19 @@ def test_decode_options_validation(L):
                 cora.decode_options(eos_id=-7)):
         rc = L.cora_session_create_ex(16, 1, z.ctypes.data, 8, 64, 32, 32, 0.5, 1, byref(opt), byref(out))
         assert rc == cora.CORA_EINVAL, (opt.schedule, opt.persistence, opt.eos_id)
+
+
+def test_unknown_weight_dtype_rejected(L):
+    cfg = dict(n_layers=1, d_model=128, n_heads=2, n_kv_heads=2, head_dim=64, ffn=64, vocab=10, mask_id=9,
+               rope_theta=1e4, norm_eps=1e-5)
+    with pytest.raises(cora.CoraError) as e:
+        cora.cora_model_create(cfg, {"embed": 16, "lm_head": 16, "dtype": 7})
+    assert e.value.code == cora.CORA_EINVAL and "dtype" in str(e.value)
+
+
+def test_denoise_step_argument_validation(L):
+    """NULL session and block/step below -1 are rejected before the session is read."""
+    assert L.cora_denoise_step(None, -1, -1, None, None, None) == cora.CORA_EINVAL
+    assert L.cora_denoise_step(16, -2, 0, None, None, None) == cora.CORA_EINVAL
+    assert L.cora_denoise_step(16, 0, -5, None, None, None) == cora.CORA_EINVAL
+    assert L.cora_session_finished(None, None) == cora.CORA_EINVAL

@@ -61,9 +61,15 @@ def test_replay_parity_every_step(tiny):
             ctrl = np.array([[st["block"], st["step"], st["passes_before"], 0]], np.int32)
             cora.cora_session_write(s, tokens=st["canvas"][None], state=st["gen_state"][None],
                                     persist=b0.persist[None], prev=b0.prev[None], ctrl=ctrl)
-            cora.cora_denoise_step(s)
+            c_step = np.full((1, BL), -1.0, np.float32)
+            a_step = np.full((1, BL), -1, np.int32)
+            d_step = np.full(1, 7, np.uint8)
+            cora.cora_denoise_step(s, st["block"], st["step"], c_step, a_step, d_step)
             out = cora.cora_session_read(s, 1, P + G, G, BL)
             c, a = out["conf"][0], out["argmax"][0]
+            # the step's own outputs are the session's Eq. 1 state and the gate's block-done flag
+            assert np.array_equal(c_step[0], c) and np.array_equal(a_step[0], a)
+            assert d_step[0] == int(not np.any(out["state"][0][st["block"] * BL:(st["block"] + 1) * BL] == 0))
             dc = np.abs(c - st["conf"])
             max_dc = max(max_dc, float(dc.max()))
             assert dc.max() <= 2e-2, (st["block"], st["step"], dc.max())
@@ -95,6 +101,51 @@ def test_replay_parity_every_step(tiny):
     finally:
         cora.cora_session_destroy(s)
     print(f"replayed {len(tr.steps)} steps, {robust_steps} with flip-proof decisions, max|dc| = {max_dc:.2e}")
+
+
+def test_denoise_step_rejects_a_wrong_block_or_step(tiny):
+    """cora_denoise_step(s, block, step, ...) checks the caller's (block, step)
+    against the session before launching: a mismatch is CORA_ESTATE and
+    leaves the state untouched; -1 skips the check."""
+    m, _, prompt = tiny
+    s = cora.cora_session_create(m, 1, prompt[:1], P, G, BL, T, TAU, K)
+    try:
+        cora.cora_denoise_step(s, 0, 0)
+        before = cora.cora_session_read(s, 1, P + G, G, BL)
+        assert before["ctrl"][0, :3].tolist() == [0, 1, 1]
+        for blk, stp in ((1, 1), (0, 0), (0, 2)):
+            with pytest.raises(cora.CoraError) as e:
+                cora.cora_denoise_step(s, blk, stp)
+            assert e.value.code == cora.CORA_ESTATE
+        after = cora.cora_session_read(s, 1, P + G, G, BL)
+        assert all(np.array_equal(before[k], after[k]) for k in before)
+        cora.cora_denoise_step(s, 0, -1)
+        cora.cora_denoise_step(s, -1, 2)
+        assert cora.cora_session_read(s, 1, P + G, G, BL)["ctrl"][0, 2] == 3
+    finally:
+        cora.cora_session_destroy(s)
+
+
+def test_fp32_weights_equal_their_bf16_rounding(tiny):
+    """The tiny model's weights are fp32; the library rounds them to bf16 on
+    the device (round to nearest even).  A model built from the host-rounded
+    bf16 bits decodes to the same tokens and passes, and so does one built
+    from device-resident fp32 tensors (read in place, no staging)."""
+    m, _, prompt = tiny
+    bits = {"embed": synth.f32_to_bf16_bits(synth.weight_f32(CFG, -1, synth.EMBED)),
+            "lm_head": synth.f32_to_bf16_bits(synth.weight_f32(CFG, -1, synth.LM_HEAD))}
+    for name, kind in model.KINDS.items():
+        bits[name] = [synth.f32_to_bf16_bits(synth.weight_f32(CFG, l, kind)) for l in range(CFG["n_layers"])]
+    m16 = cora.cora_model_create(CFG, bits)
+    m32d = model.create_model(CFG, on_device_fill=True)
+    try:
+        ref = cora.cora_generate(m, prompt[:2], G, BL, T, TAU, K)
+        for other in (m16, m32d):
+            got = cora.cora_generate(other, prompt[:2], G, BL, T, TAU, K)
+            assert np.array_equal(got[0], ref[0]) and np.array_equal(got[1], ref[1])
+    finally:
+        cora.cora_model_destroy(m16)
+        cora.cora_model_destroy(m32d)
 
 
 def test_gate_off_runs_full_horizon(tiny):

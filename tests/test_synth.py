@@ -41,3 +41,22 @@ def test_gate_inputs_shapes():
     assert 0.75 < keep < 0.86
     lg = synth.gate_logits_bf16(1, 2, 32, 1000, h[-1])
     assert lg.shape == (2, 32, 1000) and lg.dtype == np.uint16
+
+
+def test_fp32_weights_are_the_unrounded_product():
+    """fp32-weight workloads keep X * scale; the bf16 workloads' values are its rounding."""
+    key = synth.stream_key(0, synth.tensor_stream(0, synth.WQ))
+    f = synth.normal_f32(key, 0, 50000, 0.02)
+    assert f.dtype == np.float32
+    assert np.array_equal(synth.normal_bf16_bits(key, 0, 50000, 0.02), synth.f32_to_bf16_bits(f))
+    b = synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(f))
+    assert np.mean(b != f) > 0.95                       # almost none is bf16-representable
+    rel = np.abs(b - f) / np.abs(f)
+    assert rel.max() <= 2.0 ** -8 + 1e-12                # bf16 rounding: half an ulp, 8 significand bits
+    cfg = dict(n_layers=1, d_model=8, n_heads=2, n_kv_heads=1, head_dim=4, ffn=12, vocab=16, mask_id=15,
+               init_sigma=0.5, head_sigma=1.5, seed=7)
+    w16 = synth.weight_f64(cfg, 0, synth.WQ)
+    w32 = synth.weight_f64(dict(cfg, weight_dtype="f32"), 0, synth.WQ)
+    assert np.array_equal(synth.f32_to_bf16_bits(w32.astype(np.float32)),
+                          synth.f32_to_bf16_bits(w16.astype(np.float32)))
+    assert not np.array_equal(w16, w32)

@@ -6,7 +6,8 @@ their loop must not enter the allocator): its scratch is a fixed array
 inside the library.  This test calls it through the C ABI twice in a row
 (the second call reuses the array the first one left behind) and compares
 each result with cora_reduce_top1 on the same logits, within the tolerance
-the other Eq. 1 tests use.  It lives in its own file, collected last.
+the other Eq. 1 tests use, and checks that the device's free memory does not
+change across the second call.  It lives in its own file, collected last.
 """
 
 import numpy as np
@@ -33,13 +34,22 @@ def test_noalloc_matches_regular_reduction_twice(rows, V):
     ref_a = torch.empty(rows, dtype=torch.int32, device="cuda")
     cora.cora_reduce_top1(lg, rows, V, ref_c, ref_a)
     rc, ra = ref_c.cpu().numpy(), ref_a.cpu().numpy()
-    for _ in range(2):
-        c = torch.full((rows,), -1.0, dtype=torch.float32, device="cuda")
-        a = torch.full((rows,), -1, dtype=torch.int32, device="cuda")
+    outs = [(torch.empty(rows, dtype=torch.float32, device="cuda"), torch.empty(rows, dtype=torch.int32, device="cuda"))
+            for _ in range(2)]
+    free = []
+    for c, a in outs:
+        c.fill_(-1.0)
+        a.fill_(-1)
+        torch.cuda.synchronize()
+        free.append(torch.cuda.mem_get_info()[0])        # cudaMemGetInfo before the call
         cora.cora_reduce_top1_noalloc(lg, rows, V, c, a)
         torch.cuda.synchronize()
+        free.append(torch.cuda.mem_get_info()[0])        # ... and after it
         assert np.array_equal(a.cpu().numpy(), ra)
         assert np.all(np.abs(c.cpu().numpy() - rc) <= 1e-4 * rc + 1e-7)
+    # The first call on a device may load the library part holding the fixed
+    # array (lazy module loading); the second call reserves no device memory.
+    assert free[2] == free[3], (free[2], free[3])
 
 
 def test_noalloc_rejects_rows_beyond_the_fixed_scratch():
