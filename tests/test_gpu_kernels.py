@@ -177,6 +177,27 @@ def test_attention(B, S, Hq, Hkv, hd):
     assert np.abs(got - ref).max() <= atol + 1e-2 * np.abs(ref).max()
 
 
+# Queries from an offset on (the rows a prefix-cache pass recomputes) against
+# every key, with enough (sequence, head, query tile) items to run the
+# persistent kernel (more items than SMs: 256, 320 and 448 here), a query
+# start that is not a multiple of the tile, and ragged last tiles.
+@pytest.mark.parametrize("B,S,Hq,Hkv,q_start", [(2, 1000, 32, 8, 488), (2, 1000, 32, 32, 480),
+                                                (4, 544, 28, 4, 96), (1, 600, 8, 2, 32)])
+def test_attention_query_rows(B, S, Hq, Hkv, q_start):
+    hd = 128
+    q_len = S - q_start
+    W = (Hq + 2 * Hkv) * hd
+    qkv = bits(6, 12, (B * S, W), 1.0)
+    out = torch.zeros((B * q_len, Hq * hd), dtype=torch.int16, device="cuda")
+    cora.cora_op_attention_rows(dev(qkv), out, B, S, Hq, Hkv, hd, q_start, q_len)
+    x = f64(qkv).reshape(B, S, Hq + 2 * Hkv, hd)
+    ref = np.stack([O.attention(x[b, :, :Hq], x[b, :, Hq: Hq + Hkv], x[b, :, Hq + Hkv:])[q_start:]
+                    for b in range(B)])
+    got = from_dev_bf16(out).reshape(B, q_len, Hq, hd)
+    atol = 1e-2 * np.sqrt(np.mean(ref ** 2))
+    assert np.abs(got - ref).max() <= atol + 1e-2 * np.abs(ref).max()
+
+
 # ---------------------------------------------------------------- LM head
 @pytest.mark.parametrize("R,V,d", [(32, 2048, 256), (5, 1000, 128), (256, 4096, 512), (128, 1088, 256),
                                    (32, 40000, 4096)])
