@@ -47,7 +47,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # changed, and for workloads without a capture.
 NCU_TRAFFIC = {
     # gemm_tc2_kernel, mean of the QKV / O / gate-up / down launches (read + write):
-    # (124.4 + 46.3 + 245.1 + 125.6) MB / 4, profiles/gemm_tc2_llada8b_256.md
+    # (124.4 + 46.3 + 245.1 + 125.6) MB / 4
     ("gemm", "d8e0704d8d40", "llada8b-shape-256+256"): 135_355_000,
 }
 
@@ -251,21 +251,34 @@ def tiny_leg(reps: int = 5):
                              "tokens_per_s": round(G / ora_s, 2), "sample": "the whole decode of the same prompt"}}
 
 
+def flush_l2(buf):
+    """Evicts L2 by reading a 1 GiB buffer (a reduction: L2 ends up holding clean
+    lines of it, so the timed kernel's reads evict without write-backs).  It
+    runs ~0.15 ms on the GPU, long enough for the host to queue the timed
+    launch before the start event is reached."""
+    import torch
+    buf.view(torch.int64).sum()
+
+
 def gate_isolation(peaks, reps: int = 5, with_oracle: bool = False):
     """Eq. 1 from materialised bf16 logits [B, 32, 126464] + transfer rule +
-    gate (cora_reduce_gate), B in {1, 8, 64}; HBM-bound.  L2 is flushed
-    (a 256 MB write) before every timed launch; CUDA events bracket the launch
-    only.  With ``with_oracle`` the oracle's reduction + gate on the same
-    logits and state is timed on the host as the CPU baseline (float64 numpy,
-    the library's default thread count; the bf16 -> float32 widening of the
-    logits is outside the timing)."""
+    gate (cora_reduce_gate), B in {1, 8, 64}; HBM-bound.  Every timed launch
+    starts from the workload's configured state: the persistence counters and
+    previous predictions that the seeded 8-step argmax history leaves (run
+    through the library's own gate with k = 0 and the gate off, so only Eq. 2
+    acts), then half of the positions marked resolved.  The state is restored
+    and L2 flushed (a 1 GiB read) before every timed launch; CUDA events
+    bracket the launch only.  With ``with_oracle`` the oracle's reduction +
+    gate on the same logits and state is timed on the host as the CPU baseline
+    (float64 numpy, the library's default thread count; the bf16 -> float32
+    widening of the logits is outside the timing)."""
     import torch
 
     from paper_2608_11235_gb300 import configs, cora, synth
 
     gi = configs.GATE_ISOLATION
     R, V = gi["rows"], gi["vocab"]
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    flush = torch.zeros(1 << 30, dtype=torch.uint8, device="cuda")
     out = {}
     for B in gi["batches"]:
         hist = synth.gate_history(gi["seed"], B, R, V, gi["n_hist"], gi["keep"])
@@ -275,12 +288,24 @@ def gate_isolation(peaks, reps: int = 5, with_oracle: bool = False):
         conf, arg, prev, persist = st(torch.float32), st(torch.int32), st(torch.int32), st(torch.int32)
         state, tokens, unmask, accept = st(torch.uint8), st(torch.int32), st(torch.uint8), st(torch.uint8)
         done = torch.zeros(B, dtype=torch.uint8, device="cuda")
+        # Eq. 2 over the history on the GPU: every position unresolved, k = 0, gate off
+        prev.fill_(-1)
+        for t in range(hist.shape[0]):
+            h = torch.from_numpy(np.ascontiguousarray(hist[t]).astype(np.int32)).cuda()
+            cora.cora_gate_transfer(conf, h, prev, persist, state, tokens, B, R, 0, 2.0, -1, unmask, accept, done)
+        unresolved = torch.from_numpy(synth.gate_unresolved(gi["seed"], B, R, gi["masked_frac"])).cuda()
+        alt = (1 + torch.arange(B * R, device="cuda").reshape(B, R) % 2).to(torch.uint8)
+        state0 = torch.where(unresolved, torch.zeros_like(state), alt)
+        tokens0 = torch.where(unresolved, torch.full_like(tokens, V - 1),
+                              torch.from_numpy(hist[-1].astype(np.int32)).cuda())
+        prev0, persist0 = prev.clone(), persist.clone()
         ts = []
         for i in range(reps + 2):
-            flush.fill_(i & 0xFF)
-            prev.fill_(-1)
-            persist.zero_()
-            state.zero_()
+            prev.copy_(prev0)
+            persist.copy_(persist0)
+            state.copy_(state0)
+            tokens.copy_(tokens0)
+            flush_l2(flush)  # ~0.15 ms on the GPU: the launch below is queued before e0 is reached
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record()
             cora.cora_reduce_gate(lg, B, R, V, conf, arg, prev, persist, state, tokens, gi["k_step"], gi["tau"],
@@ -293,18 +318,22 @@ def gate_isolation(peaks, reps: int = 5, with_oracle: bool = False):
         nbytes = B * R * V * 2
         gbs = nbytes / (ms * 1e-3) / 1e9
         out[f"B{B}"] = {"us": round(ms * 1e3, 2), "GB_s": round(gbs, 1),
-                        "frac": round(gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]), 4), "bytes": nbytes}
-        del lg
+                        "frac": round(gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]), 4), "bytes": nbytes,
+                        "state": f"{gi['n_hist']}-step argmax history, {int(100 * gi['masked_frac'])} % masked",
+                        "accepted": int(accept.sum().item()), "transferred": int(unmask.sum().item())}
         if with_oracle:
             from oracle import cora_oracle as O
             lf = synth.bf16_bits_to_f32(lg_host)
-            z = np.zeros((B, R), np.int64)
+            s0 = state0.cpu().numpy()
+            t0n = tokens0.cpu().numpy().astype(np.int64)
+            p0 = persist0.cpu().numpy().astype(np.int64)
+            v0 = prev0.cpu().numpy().astype(np.int64)
             t0 = time.perf_counter()
-            O.reduce_and_gate(lf, z, z.astype(np.uint8), z, np.full((B, R), -1, np.int64), gi["k_step"], gi["tau"],
-                              gi["K"])
+            O.reduce_and_gate(lf, t0n, s0, p0, v0, gi["k_step"], gi["tau"], gi["K"])
             dt = time.perf_counter() - t0
             out[f"B{B}"]["cpu_baseline"] = {"kind": "oracle", "us": round(dt * 1e6, 1),
                                             "GB_s": round(nbytes / dt / 1e9, 3)}
+        del lg
     return out
 
 
@@ -312,13 +341,14 @@ def attention_shapes(peaks, reps: int = 5):
     """The attention kernel alone at the attention shape of each 8B-class
     workload (batch, canvas length, heads as configured; seeded N(0, 1) bf16
     Q/K/V from the device generator).  FLOPs per launch 4 B Hq S^2 hd against
-    the burst bf16 peak (a kernel timed in isolation).  L2 is flushed (a 256 MB
-    write) before every timed launch; CUDA events bracket the launch only."""
+    the burst bf16 peak (a kernel timed in isolation).  L2 is flushed (a 1 GiB
+    read, long enough that the launch is queued before e0 is reached) before
+    every timed launch; CUDA events bracket the launch only."""
     import torch
 
     from paper_2608_11235_gb300 import configs, cora, synth
 
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    flush = torch.zeros(1 << 30, dtype=torch.uint8, device="cuda")
     peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
     out = {}
     for name in ("llada8b-shape-256+256", "dream7b-shape-256+512-b4", "llada8b-shape-512+1024-b8"):
@@ -331,7 +361,7 @@ def attention_shapes(peaks, reps: int = 5):
         cora.cora_synth_normal_bf16(qkv, n, synth.stream_key(23, 1), 0, float(synth.normal_scale_f32(1.0)))
         ts = []
         for i in range(reps + 2):
-            flush.fill_(i & 0xFF)
+            flush_l2(flush)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record()
             cora.cora_op_attention(qkv, o, B, S, hq, hkv, hd)
@@ -345,6 +375,125 @@ def attention_shapes(peaks, reps: int = 5):
                      "achieved": round(tf, 1), "unit": "TFLOP/s", "peak": peak, "frac": round(tf / peak, 4)}
         del qkv, o
     out["peak_source"] = "bf16 burst (kernel timed alone)"
+    return out
+
+
+def profile_pass(cora, s, cfg, prompt_dev):
+    """Per-launch device times of the first pass of a decode, two eager runs
+    (CUDA events around every launch on the session's stream), the smaller
+    time of each launch kept: {kind: [ms, ...]}."""
+    cora.cora_session_reset(s, prompt_dev)
+    prof = cora.cora_session_profile_step(s, cfg["n_layers"])
+    cora.cora_session_reset(s, prompt_dev)
+    prof2 = cora.cora_session_profile_step(s, cfg["n_layers"])
+    by = {}
+    for (k1, t1), (_, t2) in zip(prof, prof2):
+        by.setdefault(k1, []).append(min(t1, t2))
+    return by
+
+
+def pass_rooflines(cora, s, cfg, prompt_dev, peaks, peak_src):
+    """(roofline of the dominant GEMM kernel, per-kernel shares, LM head and
+    attention rooflines) of one dense pass of workload ``cfg``."""
+    by = profile_pass(cora, s, cfg, prompt_dev)
+    costs = kernel_costs(cfg)
+    gemm_kinds = ["gemm_qkv_rope", "gemm_o_resid", "gemm_gate_up_swiglu", "gemm_down_resid"]
+    gemm_ms = sum(sum(by[k]) for k in gemm_kinds)
+    gemm_flops = sum(costs[k] * len(by[k]) for k in gemm_kinds)
+    n_gemm = sum(len(by[k]) for k in gemm_kinds)
+    step_ms = sum(sum(v) for v in by.values())
+    gemm_tflops = gemm_flops / (gemm_ms * 1e-3) / 1e12
+    peak_tf = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    hbm = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    head_ms = sum(by["lm_head_top1"]) / len(by["lm_head_top1"])
+    head_gbs = costs["lm_head_top1_bytes"] / (head_ms * 1e-3) / 1e9
+    attn_ms = sum(by["attention"]) / len(by["attention"])
+    kernels = {k: {"launches_per_pass": len(v), "ms_per_launch": round(sum(v) / len(v), 5),
+                   "share": round(sum(v) / step_ms, 4)} for k, v in sorted(by.items())}
+    traffic = NCU_TRAFFIC.get(("gemm", src_hash("gemm.cu"), cfg["name"]))  # per workload: the shapes differ
+    roofline = {"bound": "tensor", "kernel": "gemm_tc2_kernel (QKV+RoPE, O+res, gate/up+SwiGLU, down+res)",
+                "achieved": round(gemm_tflops, 2), "peak": peak_tf, "unit": "TFLOP/s",
+                "frac": round(gemm_tflops / peak_tf, 4), "traffic": traffic,
+                "peak_source": f"{peak_src} bf16 sustained", "flops_per_launch": round(gemm_flops / n_gemm),
+                "ms_per_launch": round(gemm_ms / n_gemm, 5)}
+    others = {
+        "lm_head_top1": {"bound": "hbm", "achieved": round(head_gbs, 1), "unit": "GB/s", "peak": hbm,
+                         "frac": round(head_gbs / hbm, 4),
+                         "bytes_per_launch": costs["lm_head_top1_bytes"], "ms_per_launch": round(head_ms, 5)},
+        "attention": {"bound": "tensor", "kernel": attn_kernel_name(cfg),
+                      "achieved": round(costs["attention"] / (attn_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s",
+                      "peak": peak_tf, "frac": round(costs["attention"] / (attn_ms * 1e-3) / 1e12 / peak_tf, 4),
+                      "ms_per_launch": round(attn_ms, 5)},
+        "pass_model_tflops": round((gemm_flops + costs["attention"] * len(by["attention"]) +
+                                    costs["lm_head_top1_flops"]) / (step_ms * 1e-3) / 1e12, 2),
+        "eager_pass_ms": round(step_ms, 3),
+    }
+    return roofline, kernels, others
+
+
+def timed_decode(cora, torch, m, cfg, prompt_dev, tau, K, opt=None, warm_steps=2):
+    """One complete decode of ``cfg``'s batch through a fresh session, timed
+    with CUDA events on the session's stream (device-resident prompt): the
+    session is created (graphs captured), warmed by ``warm_steps`` executed
+    steps, reset, then cora_session_run runs the whole decode.  Returns
+    (session, ms, batched passes, per-sequence passes)."""
+    B, P, G, BL, T = cfg["batch"], cfg["prompt_len"], cfg["gen_len"], cfg["block_len"], cfg["steps_per_block"]
+    s = cora.cora_session_create(m, B, prompt_dev, P, G, BL, T, tau, K, options=opt)
+    stream = torch.cuda.ExternalStream(cora.cora_session_stream(s))
+    for _ in range(warm_steps):
+        if cora.cora_denoise_step(s):
+            break
+    cora.cora_session_reset(s, prompt_dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    steps, _ = cora.cora_session_run(s)
+    e1.record(stream)
+    e1.synchronize()
+    carry = opt is not None and opt.persistence == cora.PERSIST_CARRY  # Eq. 1 state on every generation row
+    ctrl = cora.cora_session_read(s, B, P + G, G, BL, eq1_rows=G if carry else BL)["ctrl"]
+    return s, e0.elapsed_time(e1), steps, ctrl[:, 2].astype(np.int64)
+
+
+def workload_leg(name, peaks, peak_src, m_same=None):
+    """A further 8B-class workload (the Dream-shaped batch of 4, or the
+    fixed-horizon 512 + 1024 batch of 8): one complete decode with the
+    configured N(0, 0.02) head and one with the gate-exercising head, each
+    timed with CUDA events; executed passes per sequence against the horizon;
+    GEMM and attention rooflines of its dense pass.  ``m_same``: a model
+    handle with this workload's weights already resident (reused for the
+    configured head)."""
+    import torch
+
+    from paper_2608_11235_gb300 import configs, cora, model, synth
+
+    cfg = dict(configs.PRESETS[name])
+    B, P, G, BL, T = cfg["batch"], cfg["prompt_len"], cfg["gen_len"], cfg["block_len"], cfg["steps_per_block"]
+    horizon = (G // BL) * T
+    out = {"workload": name, "batch": B, "prompt_len": P, "gen_len": G, "block_len": BL, "steps_per_block": T,
+           "tau": cfg["tau"], "K": cfg["K"], "horizon": horizon,
+           "timing": "CUDA events on the session stream around one complete decode (one graph launch), "
+                     "device-resident prompt; weights larger than L2"}
+    for variant in ("as_configured", "gate_exercising"):
+        c = cfg if variant == "as_configured" else configs.gate_exercising(cfg)
+        own = not (variant == "as_configured" and m_same is not None)
+        m = model.create_model(c) if own else m_same
+        try:
+            prompt_dev = torch.from_numpy(synth.prompts(c["prompt_seed"], B, P, c["mask_id"])).cuda()
+            s, ms, batched, passes = timed_decode(cora, torch, m, c, prompt_dev, c["tau"], c["K"])
+            try:
+                roof, kern, others = pass_rooflines(cora, s, c, prompt_dev, peaks, peak_src)
+            finally:
+                cora.cora_session_destroy(s)
+        finally:
+            if own:
+                cora.cora_model_destroy(m)
+        out[variant] = {"head_sigma": round(c["head_sigma"], 6), "tokens_per_s": round(B * G / (ms * 1e-3), 3),
+                        "ms_per_decode": round(ms, 1), "batched_passes": int(batched),
+                        "passes_per_seq": passes.tolist(), "passes_per_block": round(float(passes.mean()) / (G // BL), 3),
+                        "rho": round(float(passes.mean()) / horizon, 4), "ms_per_batched_pass": round(ms / batched, 3),
+                        "roofline": roof, "attention": others["attention"], "lm_head_top1": others["lm_head_top1"],
+                        "pass_model_tflops": others["pass_model_tflops"],
+                        "kernel_shares": {k: v["share"] for k, v in kern.items()}}
     return out
 
 
@@ -422,44 +571,7 @@ def run_cora(args, cfg, ws, rank, local):
               "timing": "CUDA events on the session stream, device-resident prompt"}
 
     # ----- per-kernel device times (one eager pass with events around each launch)
-    cora.cora_session_reset(s, prompt_dev)
-    prof = cora.cora_session_profile_step(s, cfg["n_layers"])
-    cora.cora_session_reset(s, prompt_dev)
-    prof2 = cora.cora_session_profile_step(s, cfg["n_layers"])
-    by = {}
-    for (k1, t1), (_, t2) in zip(prof, prof2):
-        by.setdefault(k1, []).append(min(t1, t2))
-    costs = kernel_costs(cfg)
-    gemm_kinds = ["gemm_qkv_rope", "gemm_o_resid", "gemm_gate_up_swiglu", "gemm_down_resid"]
-    gemm_ms = sum(sum(by[k]) for k in gemm_kinds)
-    gemm_flops = sum(costs[k] * len(by[k]) for k in gemm_kinds)
-    n_gemm = sum(len(by[k]) for k in gemm_kinds)
-    step_ms = sum(sum(v) for v in by.values())
-    gemm_tflops = gemm_flops / (gemm_ms * 1e-3) / 1e12
-    peak_tf = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-    head_ms = sum(by["lm_head_top1"]) / len(by["lm_head_top1"])
-    head_gbs = costs["lm_head_top1_bytes"] / (head_ms * 1e-3) / 1e9
-    attn_ms = sum(by["attention"]) / len(by["attention"])
-    kernels = {k: {"launches_per_pass": len(v), "ms_per_launch": round(sum(v) / len(v), 5),
-                   "share": round(sum(v) / step_ms, 4)} for k, v in sorted(by.items())}
-    traffic = NCU_TRAFFIC.get(("gemm", src_hash("gemm.cu"), cfg["name"]))  # per workload: the shapes differ
-    roofline = {"bound": "tensor", "kernel": "gemm_tc2_kernel (QKV+RoPE, O+res, gate/up+SwiGLU, down+res)",
-                "achieved": round(gemm_tflops, 2), "peak": peak_tf, "unit": "TFLOP/s",
-                "frac": round(gemm_tflops / peak_tf, 4), "traffic": traffic,
-                "peak_source": f"{peak_src} bf16 sustained", "flops_per_launch": round(gemm_flops / n_gemm),
-                "ms_per_launch": round(gemm_ms / n_gemm, 5)}
-    others = {
-        "lm_head_top1": {"bound": "hbm", "achieved": round(head_gbs, 1), "unit": "GB/s",
-                         "peak": peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]),
-                         "frac": round(head_gbs / peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"]), 4),
-                         "bytes_per_launch": costs["lm_head_top1_bytes"], "ms_per_launch": round(head_ms, 5)},
-        "attention": {"bound": "tensor", "kernel": attn_kernel_name(cfg),
-                      "achieved": round(costs["attention"] / (attn_ms * 1e-3) / 1e12, 2), "unit": "TFLOP/s",
-                      "peak": peak_tf, "frac": round(costs["attention"] / (attn_ms * 1e-3) / 1e12 / peak_tf, 4),
-                      "ms_per_launch": round(attn_ms, 5)},
-        "pass_model_tflops": round((gemm_flops + costs["attention"] * len(by["attention"]) +
-                                    costs["lm_head_top1_flops"]) / (step_ms * 1e-3) / 1e12, 2),
-    }
+    roofline, kernels, others = pass_rooflines(cora, s, cfg, prompt_dev, peaks, peak_src)
 
     # ----- end to end through the public call, host buffers (pinned), copies inside
     prompt_pin = torch.from_numpy(prompt).pin_memory()
@@ -477,49 +589,48 @@ def run_cora(args, cfg, ws, rank, local):
     if not args.no_variant:
         cfg_g = configs.gate_exercising(cfg)
         cora.cora_session_destroy(s)
+        s = None
         mg = model.create_model(cfg_g, device=f"cuda:{local}")
-        cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau, K)
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        reps = max(1, args.steps)
-        for _ in range(reps):
-            _, pg, bg = cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau, K)
-        tg = time.perf_counter() - t0
-        gx = {"head_sigma": round(cfg_g["head_sigma"], 6), "tokens_per_s": round(B * G * reps / tg, 2),
+        sg, msg, _, pg = timed_decode(cora, torch, mg, cfg_g, prompt_dev, tau, K)
+        cora.cora_session_destroy(sg)
+        gx = {"head_sigma": round(cfg_g["head_sigma"], 6), "tokens_per_s": round(B * G / (msg * 1e-3), 2),
               "passes_per_block": round(float(pg.mean()) / (G // BL), 3),
-              "rho": round(float(pg.mean()) / ((G // BL) * T), 4), "timing": "host wall clock, e2e call"}
+              "rho": round(float(pg.mean()) / ((G // BL) * T), 4),
+              "timing": "CUDA events on the session stream around one complete decode (device-resident prompt)"}
         # (tau, K, schedule) sweep on the same model: the gate's operating
-        # points and the remaining-steps schedule (one warm call, one timed)
-        # dense endpoint Y* of the same prompts (gate off), for the disagreement columns
-        sd = cora.cora_session_create(mg, B, prompt_pin.numpy(), P, G, BL, T, 2.0, K)
+        # points and the remaining-steps schedule, each one decode timed with
+        # CUDA events; the dense endpoint Y* of the same prompts (gate off)
+        # gives the disagreement columns
+        sd = cora.cora_session_create(mg, B, prompt_dev, P, G, BL, T, 2.0, K)
         cora.cora_session_run(sd)
         sweep = []
         for tau_s, K_s, sched, pers in ((tau, K, 0, 0), (tau, 0, 0, 0), (tau, 2, 0, 0), (0.9, K, 0, 0),
                                         (0.5, K, 0, 0), (tau, K, 1, 0), (tau, K, 0, 1), (2.0, K, 0, 0)):
             opt = cora.decode_options(schedule=sched, persistence=pers)
-            cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau_s, K_s, options=opt)
-            t0 = time.perf_counter()
-            _, ps, _ = cora.cora_generate(mg, prompt_pin.numpy(), G, BL, T, tau_s, K_s, options=opt)
-            dt = time.perf_counter() - t0
-            sv = cora.cora_session_create(mg, B, prompt_pin.numpy(), P, G, BL, T, tau_s, K_s, options=opt)
-            cora.cora_session_run(sv)
+            sv, dt_ms, _, ps = timed_decode(cora, torch, mg, cfg_g, prompt_dev, tau_s, K_s, opt=opt)
             n_acc, n_ad, n_od = cora.cora_session_disagreement(sv, sd, B)
             cora.cora_session_destroy(sv)
             sweep.append({"tau": tau_s, "K": K_s, "schedule": "remaining" if sched else "fixed",
                           "persistence": "carry" if pers else "block",
                           "passes_per_block": round(float(ps.mean()) / (G // BL), 3),
                           "rho": round(float(ps.mean()) / ((G // BL) * T), 4),
-                          "tokens_per_s": round(B * G / dt, 2),
+                          "tokens_per_s": round(B * G / (dt_ms * 1e-3), 2),
                           "accepted_per_seq": float(n_acc.mean()),
                           "L_acc": round(float(np.mean(n_ad / np.maximum(1, n_acc))), 4),
                           "L_out": round(float(np.mean(n_od / G)), 4)})
         cora.cora_session_destroy(sd)
         gx["sweep"] = sweep
         cora.cora_model_destroy(mg)
-        s = None
     if s is not None:
         cora.cora_session_destroy(s)
-    cora.cora_model_destroy(m)
+    workloads = None
+    if not args.no_variant and not args.no_workloads and ws == 1 and cfg["name"] == "llada8b-shape-256+256":
+        workloads = {"llada8b-shape-512+1024-b8": workload_leg("llada8b-shape-512+1024-b8", peaks, peak_src, m_same=m)}
+        cora.cora_model_destroy(m)
+        m = None
+        workloads["dream7b-shape-256+512-b4"] = workload_leg("dream7b-shape-256+512-b4", peaks, peak_src)
+    if m is not None:
+        cora.cora_model_destroy(m)
     gate_iso = None if args.no_variant else gate_isolation(
         peaks, with_oracle=(rank == 0 and ws == 1 and not args.no_cpu_baseline))
     tiny = None if args.no_variant else tiny_leg()
@@ -557,6 +668,7 @@ def run_cora(args, cfg, ws, rank, local):
         "gate_isolation": gate_iso,
         "tiny": tiny,
         "attention_shapes": attn_shapes,
+        "workloads": workloads,
     }
     return result, float(per_seq_passes.mean())
 
@@ -570,6 +682,8 @@ def main():
     ap.add_argument("--workload", default="llada8b-shape-256+256")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-variant", action="store_true")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the Dream-shaped and 512+1024 x 8 decodes (about four minutes)")
     ap.add_argument("--layers", type=int, default=0, help="override n_layers (same per-launch shapes)")
     args = ap.parse_args()
     from paper_2608_11235_gb300 import configs

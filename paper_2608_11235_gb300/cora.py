@@ -246,8 +246,9 @@ def cora_session_disagreement(session, dense, B):
 
 
 def cora_session_read(session, B, S, G, BL, eq1_rows=None) -> dict:
-    """eq1_rows: rows of persist/prev/conf/argmax per sequence (BL, or G for a
-    carry-over persistence session)."""
+    """eq1_rows: rows of persist/prev/conf/argmax per sequence: BL, or G for a
+    carry-over persistence session (the library writes B * G entries there,
+    so a smaller buffer would be overrun)."""
     E = BL if eq1_rows is None else eq1_rows
     out = dict(tokens=np.zeros((B, S), np.int32), state=np.zeros((B, G), np.uint8),
                persist=np.zeros((B, E), np.int32), prev=np.zeros((B, E), np.int32),
