@@ -210,13 +210,13 @@ def attn_kernel_name(cfg: dict) -> str:
     """The attention kernel a dense pass of this workload launches: head_dim 64
     runs the mma.sync kernel; head_dim 128 runs one CTA per (sequence, head,
     128-query tile) item while the items fit on the SMs, else the persistent
-    kernel."""
+    two-query-tile kernel."""
     if cfg["head_dim"] != 128:
         return "attention_kernel"
     import torch
     items = -(-(cfg["prompt_len"] + cfg["gen_len"]) // 128) * cfg["n_heads"] * cfg["batch"]
     sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
-    return "attention_tc_kernel" if items <= sms else "attention_tc_persistent_kernel"
+    return "attention_tc_kernel" if items <= sms else "attention_tc2_kernel"
 
 
 def tiny_leg(reps: int = 5):

@@ -1,10 +1,9 @@
 // Bidirectional (non-causal) attention on the 5th-generation tensor cores,
-// head_dim 128.  Work item = (sequence, query head, 128-query tile).  Two
-// kernels share the per-tile pipeline below: attention_tc_kernel runs one
-// item per CTA (when the items fit on the SMs at once), and
-// attention_tc_persistent_kernel loops each CTA over several items (when
-// there are more items than SMs).  Keys and values stream through shared
-// memory in 128-key tiles (TMA, double-buffered).
+// head_dim 128.  Work item = (sequence, query head, 128-query tile).
+// attention_tc_kernel runs one item per CTA and serves launches whose items
+// fit on the SMs at once; launches with more items than SMs go to the
+// two-query-tile persistent kernel (attention_tc2.cu).  Keys and values
+// stream through shared memory in 128-key tiles (TMA, double-buffered).
 //
 // Per key tile j:
 //   S_j = Q K_j^T        tcgen05.mma M=128 (queries) x N=128 (keys) x K=128 (hd), TMEM
@@ -21,8 +20,7 @@
 // P <= 2^8 keeps full bf16 precision, so the result is unchanged while the
 // softmax warps never wait for a PV in the common case.
 // Two TMEM buffers for S and two P buffers let the softmax of tile j overlap
-// the MMAs of tiles j-1 and j+1.  TMEM: S[0] +0, S[1] +128, O +256 (the
-// persistent kernel alternates items between O[0] +256 and O[1] +384).
+// the MMAs of tiles j-1 and j+1.  TMEM: S[0] +0, S[1] +128, O +256.
 // K and V buffers are released separately (K_j once QK_j is done, V_j once
 // PV_j is), so K_{j+2} streams in while tile j is still in the softmax.
 // Warps: 0 = TMA producer, 1 = TMEM allocator + MMA issuer, 2..5 = softmax and
@@ -104,9 +102,8 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void*
 }
 
 // One CTA per item (grid = query tiles x heads x sequences): used when the
-// items fit on the SMs at once.  It keeps no state across items and compiles
-// to fewer registers (196 against 215); on 128 items at S = 512 it measured
-// 12.6 us against 13.5 us for the persistent kernel (ncu, same command).
+// items fit on the SMs at once.  (On 128 items at S = 512 it measured 12.6 us
+// against 13.5 us for a persistent one-tile-per-item variant, ncu, same command.)
 __global__ void __launch_bounds__(192, 1)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ CUtensorMap tmOut, int S,
                         int Hq, int Hkv, int q_start, int* err) {
@@ -361,339 +358,12 @@ __global__ void __launch_bounds__(192, 1)
   }
 }
 
-// Persistent: min(items, SMs) CTAs, CTA c taking items c, c + grid, ...
-// (query tile fastest, so CTAs running at the same time share the same heads'
-// keys and values in L2).  Every ring slot and barrier phase counts key tiles
-// across the CTA's items, so the next item's Q (loaded once the current item's
-// last QK is done) and first K/V tiles stream in, and its first S tile is
-// computed, while the softmax warps finish the current item.  Items alternate
-// between the two O accumulators (TMEM columns 256 and 384), so an item's first
-// PV never waits for the previous item's read-out.  Used when there are more
-// items than SMs.
-__global__ void __launch_bounds__(192, 1)
-    attention_tc_persistent_kernel(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ CUtensorMap tmOut, int S,
-                        int Hq, int Hkv, int q_start, int n_qt, int n_items, int* err) {
-  using namespace attn;
-  // idesc: M = 128, N = 128, bf16 x bf16 -> f32; PV reads B (V) MN-major.
-  constexpr uint32_t IDESC_QK = idesc_bf16_f32(128, 128);
-  constexpr uint32_t IDESC_PV = idesc_bf16_f32(128, 128) | (1u << 16);
-
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem;
-  uint8_t* sK[2] = {smem + OPND, smem + 2 * OPND};
-  uint8_t* sV[2] = {smem + 3 * OPND, smem + 4 * OPND};
-  uint8_t* sP[2] = {smem + 5 * OPND, smem + 6 * OPND};
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 7 * OPND);
-  uint64_t* qfull = bars + 0;
-  uint64_t* kfull = bars + 1;    // [2] K_j landed
-  uint64_t* vfull = bars + 3;    // [2] V_j landed
-  uint64_t* kempty = bars + 5;   // [2] QK_j done with K_j
-  uint64_t* vempty = bars + 7;   // [2] PV_j done with V_j
-  uint64_t* sfull = bars + 9;    // [2] S_j in TMEM
-  uint64_t* sfree = bars + 11;   // [2] S_j read out by the four softmax warps
-  uint64_t* pfull = bars + 13;   // [2] P_j written (and O rescaled, if it was)
-  uint64_t* pdone = bars + 15;   // [2] PV_j complete (P buffer free, O up to date)
-  uint64_t* qempty = bars + 17;  // every QK of an item done (Q buffer free)
-  uint64_t* oempty = bars + 18;  // [2] O buffer read out by the four softmax warps
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 20);
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_kt = (S + KT - 1) / KT;
-  const int group = Hq / Hkv;
-  // Item -> (query tile, query head, sequence), query tile fastest.
-  auto item_coords = [&](int item, int& qt, int& h, int& b) {
-    qt = item % n_qt;
-    const int rest = item / n_qt;
-    h = rest % Hq;
-    b = rest / Hq;
-  };
-
-  if (threadIdx.x == 0) {
-    mbar_init(qfull, 1);
-    mbar_init(qempty, 1);
-    for (int i = 0; i < 2; ++i) {
-      mbar_init(&oempty[i], 4);
-      mbar_init(&kfull[i], 1);
-      mbar_init(&vfull[i], 1);
-      mbar_init(&kempty[i], 1);
-      mbar_init(&vempty[i], 1);
-      mbar_init(&sfull[i], 1);
-      mbar_init(&sfree[i], 4);
-      mbar_init(&pfull[i], 4);
-      mbar_init(&pdone[i], 1);
-    }
-    *abort_flag = 0;
-    fence_barrier_init();
-  }
-  if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tmQKV);
-    tma_prefetch_desc(&tmOut);
-  }
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, 512);
-    tmem_relinquish();
-  }
-  __syncwarp();  // converged arrival (one lane of warp 0 initialised the barriers)
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem_base = *tmem_slot;
-  pdl_trigger();
-  pdl_wait();
-
-  if (warp == 0) {
-    if (lane == 0) {
-      bool ok = true;
-      int t = 0;  // key tiles loaded so far by this CTA (ring slot t & 1)
-      for (int it = 0, item = blockIdx.x; ok && item < n_items; ++it, item += gridDim.x) {
-        int qt, h, b;
-        item_coords(item, qt, h, b);
-        const int kvh = h / group;
-        const int row_base = b * S;        // first row of this sequence in [B*S, .]
-        const int q0 = q_start + qt * QT;  // queries q_start .. ; output rows relative to q_start
-        const int qcol = h * HD, kcol = (Hq + kvh) * HD, vcol = (Hq + Hkv + kvh) * HD;
-        // The Q buffer is free once every QK of the previous item has completed.
-        if (it > 0 && !mbar_wait(qempty, (it - 1) & 1, abort_flag, err, CORA_DERR_TMA_WAIT)) break;
-        mbar_arrive_expect_tx(qfull, OPND);
-        tma_load_2d(sQ, &tmQKV, qfull, qcol, row_base + q0);
-        tma_load_2d(sQ + OPND / 2, &tmQKV, qfull, qcol + 64, row_base + q0);
-        for (int j = 0; j < n_kt; ++j, ++t) {
-          const int s = t & 1;
-          const uint32_t ph = ((t >> 1) & 1) ^ 1u;
-          const int r = row_base + j * KT;
-          if (!mbar_wait(&kempty[s], ph, abort_flag, err, CORA_DERR_TMA_WAIT)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&kfull[s], OPND);
-          tma_load_2d(sK[s], &tmQKV, &kfull[s], kcol, r);
-          tma_load_2d(sK[s] + OPND / 2, &tmQKV, &kfull[s], kcol + 64, r);
-          if (!mbar_wait(&vempty[s], ph, abort_flag, err, CORA_DERR_TMA_WAIT)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_expect_tx(&vfull[s], OPND);
-          tma_load_2d(sV[s], &tmQKV, &vfull[s], vcol, r);
-          tma_load_2d(sV[s] + OPND / 2, &tmQKV, &vfull[s], vcol + 64, r);
-        }
-      }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      const uint32_t q_addr = smem_u32(sQ);
-      // O += P_tt V_tt for key tile tt, the jj-th tile of the CTA's item itt.
-      auto issue_pv = [&](int tt, int itt, int jj) -> bool {
-        const int s = tt & 1;
-        const uint32_t ph = (tt >> 1) & 1;
-        const int ob = itt & 1;
-        if (!mbar_wait(&pfull[s], ph, abort_flag, err, CORA_DERR_MMA_WAIT)) return false;
-        if (!mbar_wait(&vfull[s], ph, abort_flag, err, CORA_DERR_MMA_WAIT)) return false;
-        // An item's first PV overwrites its O buffer: the item two before
-        // must have been read out of it.
-        if (jj == 0 && !mbar_wait(&oempty[ob], ((itt >> 1) & 1) ^ 1u, abort_flag, err, CORA_DERR_MMA_WAIT))
-          return false;
-        tc_fence_after();
-        const uint32_t o_tmem = tmem_base + 256 + ob * 128;
-        const uint32_t p_addr = smem_u32(sP[s]), v_addr = smem_u32(sV[s]);
-#pragma unroll
-        for (int k = 0; k < KT / 16; ++k) {
-          // A = P: K-major, keys contiguous, 64-key swizzle columns 16 KB apart.
-          const uint64_t a = sw128_kmajor_desc(p_addr + (k >> 2) * (OPND / 2) + (k & 3) * 32);
-          // B = V: rows are keys (K), 64-element hd blocks 16 KB apart (MN-major).
-          const uint64_t bd = sw128_mnmajor_desc(v_addr + k * 16 * 128, OPND / 2);
-          umma_bf16(o_tmem, a, bd, IDESC_PV, (jj > 0 || k > 0) ? 1u : 0u);
-        }
-        umma_commit(&pdone[s]);
-        umma_commit(&vempty[s]);
-        return true;
-      };
-      bool ok = true;
-      int t = 0;                      // key tiles whose QK was issued
-      int tp = -1, itp = 0, jp = 0;   // the tile whose PV is still to issue
-      for (int it = 0, item = blockIdx.x; ok && item < n_items; ++it, item += gridDim.x) {
-        if (!mbar_wait(qfull, it & 1, abort_flag, err, CORA_DERR_MMA_WAIT)) {
-          ok = false;
-          break;
-        }
-        for (int j = 0; j < n_kt; ++j, ++t) {
-          const int s = t & 1;
-          const uint32_t ph = (t >> 1) & 1;
-          if (!mbar_wait(&kfull[s], ph, abort_flag, err, CORA_DERR_MMA_WAIT) ||
-              !mbar_wait(&sfree[s], ph ^ 1u, abort_flag, err, CORA_DERR_MMA_WAIT)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t k_addr = smem_u32(sK[s]);
-          const uint32_t d = tmem_base + s * 128;
-#pragma unroll
-          for (int k = 0; k < HD / 16; ++k) {
-            const uint32_t off = (k >> 2) * (OPND / 2) + (k & 3) * 32;
-            umma_bf16(d, sw128_kmajor_desc(q_addr + off), sw128_kmajor_desc(k_addr + off), IDESC_QK, k > 0);
-          }
-          umma_commit(&sfull[s]);
-          umma_commit(&kempty[s]);
-          if (j == n_kt - 1) umma_commit(qempty);
-          // The previous tile's PV (possibly the previous item's last) goes
-          // after this QK, so the QK overlaps that tile's softmax.
-          if (tp >= 0 && !issue_pv(tp, itp, jp)) {
-            ok = false;
-            break;
-          }
-          tp = t;
-          itp = it;
-          jp = j;
-        }
-      }
-      if (ok && tp >= 0) issue_pv(tp, itp, jp);
-    }
-  } else {
-    const int sub = warp & 3;
-    const int r = sub * 32 + lane;  // query row within the tile (TMEM lane)
-    const uint32_t lane_base = tmem_base + (static_cast<uint32_t>(sub * 32) << 16);
-    const float sl2 = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
-    bool ok = true;
-    int t = 0;  // key tiles this CTA's softmax has taken
-    for (int it = 0, item = blockIdx.x; ok && item < n_items; ++it, item += gridDim.x) {
-      int qt, h, b;
-      item_coords(item, qt, h, b);
-      const uint32_t o_lane = lane_base + 256 + (it & 1) * 128;
-      float m = -INFINITY, l = 0.f;
-      for (int j = 0; j < n_kt; ++j, ++t) {
-        const int s = t & 1;
-        const uint32_t ph = (t >> 1) & 1;
-        ok = mbar_wait(&sfull[s], ph, abort_flag, err, CORA_DERR_EPI_WAIT);
-        if (!ok) break;
-        tc_fence_after();
-        uint32_t v[128];
-        tmem_ld128(lane_base + s * 128, v);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sfree[s]);  // S buffer may take the tile after next
-        const int kbase = j * KT;
-        float mx8[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) mx8[i] = -INFINITY;
-        if (kbase + KT > S) {  // ragged last tile: keys past the end do not count
-#pragma unroll
-          for (int i = 0; i < KT; ++i)
-            if (kbase + i >= S) v[i] = __float_as_uint(-INFINITY);
-        }
-#pragma unroll
-        for (int i = 0; i < KT; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(v[i]));  // eight chains
-        float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                         fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-        mx *= sl2;
-        const bool raise = mx > m + kRescale;
-        if (__any_sync(0xffffffffu, raise)) {
-          const float m_new = raise ? mx : m;
-          const float a = ex2f(m - m_new);  // 0 on the first tile, 1 where not raised
-          l *= a;
-          m = m_new;
-          if (j > 0) {
-            // O holds this item's PVs up to the previous tile: wait for the
-            // last of them, then rescale in place.
-            const int tq = t - 1;
-            ok = mbar_wait(&pdone[tq & 1], (tq >> 1) & 1, abort_flag, err, CORA_DERR_EPI_WAIT);
-            if (!ok) break;
-            tc_fence_after();
-#pragma unroll 1
-            for (int c = 0; c < HD; c += 32) {
-              uint32_t o[32];
-              tmem_ld32w(o_lane + c, o);
-#pragma unroll
-              for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * a);
-              tmem_st32(o_lane + c, o);
-            }
-            tmem_wait_st();
-          }
-        }
-        // P buffer s is free once the PV of the tile two before has read it.
-        if (t >= 2) ok = mbar_wait(&pdone[s], ph ^ 1u, abort_flag, err, CORA_DERR_EPI_WAIT);
-        if (!ok) break;
-        float rs4[4] = {0.f, 0.f, 0.f, 0.f};
-        uint8_t* prow = sP[s];
-#pragma unroll
-        for (int c = 0; c < KT; c += 8) {
-          uint32_t pk[4];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            const float x0 = ex2f(fmaf(__uint_as_float(v[c + 2 * i]), sl2, -m));
-            const float x1 = ex2f(fmaf(__uint_as_float(v[c + 2 * i + 1]), sl2, -m));
-            rs4[i] += x0 + x1;
-            pk[i] = pack_bf16x2(x0, x1);
-          }
-          // keys c .. c+7 -> swizzle column c/64, 16-byte chunk (c%64)/8
-          const int chunk = (c & 63) >> 3;
-          *reinterpret_cast<uint4*>(prow + (c >> 6) * (OPND / 2) + r * 128 + ((chunk ^ (r & 7)) << 4)) =
-              make_uint4(pk[0], pk[1], pk[2], pk[3]);
-        }
-        l += (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&pfull[s]);
-      }
-      if (!ok) break;
-      // Output: wait for the item's last PV (every earlier PV is then done too,
-      // so both P buffers are free), read O and hand its TMEM buffer back,
-      // write O / l as bf16 into this warp's 32 rows of P buffer 0 (the store
-      // map's box layout) and store them by TMA.
-      const int tl = t - 1;
-      ok = mbar_wait(&pdone[tl & 1], (tl >> 1) & 1, abort_flag, err, CORA_DERR_EPI_WAIT);
-      if (!ok) break;
-      tc_fence_after();
-      uint32_t o[128];
-      tmem_ld128(o_lane, o);
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&oempty[it & 1]);
-      const float inv = 1.f / l;
-      uint8_t* stg = sP[0];
-#pragma unroll
-      for (int c = 0; c < HD; c += 8) {
-        const int chunk = (c & 63) >> 3;
-        *reinterpret_cast<uint4*>(stg + (c >> 6) * (OPND / 2) + r * 128 + ((chunk ^ (r & 7)) << 4)) = make_uint4(
-            pack_bf16x2(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
-            pack_bf16x2(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
-            pack_bf16x2(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
-            pack_bf16x2(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        for (int c = 0; c < 2; ++c)
-          tma_store_3d(&tmOut, stg + c * (OPND / 2) + sub * 32 * 128, h * HD + c * 64, qt * QT + sub * 32, b);
-        asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-        // The next item's softmax rewrites these rows of the P buffers.
-        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-      }
-      __syncwarp();
-    }
-    tc_fence_before();
-  }
-
-  // Each warp arrives converged: the producer and MMA warps ran their loops
-  // on one lane, and bar.sync counts a divergent warp's lanes separately.
-  __syncwarp();
-  tc_fence_before();
-  __syncthreads();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tmem_base, 512);
-  }
-}
-
 }  // namespace cora
 
 using namespace cora;
 
 cudaError_t attention_tc_prepare() {
-  cudaError_t e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, attn::SMEM);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attention_tc_persistent_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, attn::SMEM);
+  return cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, attn::SMEM);
 }
 
 cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
@@ -710,6 +380,6 @@ cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, 
   if (n_items <= num_sms)
     return launch_pdl(attention_tc_kernel, dim3(n_qt, Hq, B), dim3(192), attn::SMEM, st, tmQKV, tmOut, S, Hq, Hkv,
                       q_start, err);
-  return launch_pdl(attention_tc_persistent_kernel, dim3(num_sms), dim3(192), attn::SMEM, st, tmQKV, tmOut, S, Hq,
-                    Hkv, q_start, n_qt, n_items, err);
+  // More items than SMs: two query tiles per CTA (attention_tc2.cu).
+  return launch_attention_tc2(tmQKV, out, B, S, Hq, Hkv, q_start, q_len, err, num_sms, st);
 }

@@ -203,8 +203,14 @@ cudaError_t gemm_prepare();
 cudaError_t lm_head_prepare();
 cudaError_t attention_prepare();
 cudaError_t attention_tc_prepare();
+cudaError_t attention_tc2_prepare();
+// Two query tiles per CTA, persistent over (sequence, head, query-tile pair)
+// items; out bf16 [B][q_len][Hq*128] written directly.
+cudaError_t launch_attention_tc2(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
+                                 int q_len, int* err, int num_sms, cudaStream_t st);
 // tcgen05 attention for head_dim 128; tmQKV: bf16 [B*S, (Hq+2Hkv)*128], box 128 rows x 64 cols.
-// Persistent grid of min(items, num_sms) CTAs, items = ceil(q_len/128) * Hq * B.
+// Items = ceil(q_len/128) * Hq * B: one CTA per item when they fit on the SMs,
+// else the two-query-tile persistent kernel (launch_attention_tc2).
 cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
                                 int q_len, int* err, int num_sms, cudaStream_t st);
 

@@ -178,6 +178,7 @@ static int kernels_prepare() {
     CK(lm_head_prepare());
     CK(attention_prepare());
     CK(attention_tc_prepare());
+    CK(attention_tc2_prepare());
     dc->prepared = true;
   }
   return CORA_OK;
