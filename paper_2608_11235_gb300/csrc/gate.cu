@@ -71,15 +71,34 @@ __device__ __forceinline__ Top1 reduce_range(const uint16_t* __restrict__ p, int
     const uint4* pv = reinterpret_cast<const uint4*>(p);
     const int stride = blockDim.x * 8;
     int i = lo + threadIdx.x * 8;
-    for (; i + 3 * stride < hi; i += 4 * stride) {  // four 16-byte loads in flight per thread
-      const uint4 a = __ldcs(pv + (i >> 3));
-      const uint4 b = __ldcs(pv + ((i + stride) >> 3));
-      const uint4 c = __ldcs(pv + ((i + 2 * stride) >> 3));
-      const uint4 d = __ldcs(pv + ((i + 3 * stride) >> 3));
+    if (i + 3 * stride < hi) {
+      // Four 16-byte loads per batch; the next batch is loaded before the
+      // current one is reduced, so eight are in flight while the exponentials run.
+      uint4 a = __ldcs(pv + (i >> 3));
+      uint4 b = __ldcs(pv + ((i + stride) >> 3));
+      uint4 c = __ldcs(pv + ((i + 2 * stride) >> 3));
+      uint4 d = __ldcs(pv + ((i + 3 * stride) >> 3));
+      int n = i + 4 * stride;
+      for (; n + 3 * stride < hi; n += 4 * stride) {
+        const uint4 a2 = __ldcs(pv + (n >> 3));
+        const uint4 b2 = __ldcs(pv + ((n + stride) >> 3));
+        const uint4 c2 = __ldcs(pv + ((n + 2 * stride) >> 3));
+        const uint4 d2 = __ldcs(pv + ((n + 3 * stride) >> 3));
+        top1_add8(st, a, i);
+        top1_add8(st, b, i + stride);
+        top1_add8(st, c, i + 2 * stride);
+        top1_add8(st, d, i + 3 * stride);
+        a = a2;
+        b = b2;
+        c = c2;
+        d = d2;
+        i = n;
+      }
       top1_add8(st, a, i);
       top1_add8(st, b, i + stride);
       top1_add8(st, c, i + 2 * stride);
       top1_add8(st, d, i + 3 * stride);
+      i = n;
     }
     for (; i < hi; i += stride) top1_add8(st, __ldcs(pv + (i >> 3)), i);
   } else {
@@ -451,7 +470,7 @@ __global__ void step_loop_cond_kernel(cudaGraphConditionalHandle h, int32_t* sta
 using namespace cora;
 
 int reduce_top1_parts_count(int rows, int V, int num_sms) {
-  int want = (4 * num_sms + rows - 1) / rows;    // about four CTAs per SM in total
+  int want = (4 * num_sms + rows - 1) / rows;    // about four CTAs per SM in total (one wave)
   int max_chunks = (V + 4095) / 4096;            // at least 4096 elements per CTA
   int n = want < max_chunks ? want : max_chunks;
   return n < 1 ? 1 : n;
