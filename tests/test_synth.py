@@ -60,3 +60,14 @@ def test_fp32_weights_are_the_unrounded_product():
     assert np.array_equal(synth.f32_to_bf16_bits(w32.astype(np.float32)),
                           synth.f32_to_bf16_bits(w16.astype(np.float32)))
     assert not np.array_equal(w16, w32)
+
+
+def test_torch_restatement_of_the_generator_matches():
+    """The float32 bf16-point reference's torch generator (int64 wrap-around
+    arithmetic) gives synth's bits, on the CPU here and on the GPU in its own test."""
+    import bf16_emulation as E
+    for seed, stream, start, n, sigma in ((2, 0x103, 0, 5000, 0.02), (11, 2, 7_777_777_777, 3000, 8 / 64.0),
+                                          (0, 1, (1 << 40) + 3, 2000, 0.5)):
+        key = synth.stream_key(seed, stream)
+        got = E.normal_bf16(key, start, n, sigma, "cpu").view(torch.int16).numpy().view(np.uint16)
+        assert np.array_equal(got, synth.normal_bf16_bits(key, start, n, sigma))
