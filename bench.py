@@ -207,16 +207,15 @@ def kernel_costs(cfg: dict):
 
 
 def attn_kernel_name(cfg: dict) -> str:
-    """The attention kernel a dense pass of this workload launches: head_dim 64
-    runs the mma.sync kernel; head_dim 128 runs one CTA per (sequence, head,
-    128-query tile) item while the items fit on the SMs, else the persistent
-    two-query-tile kernel."""
+    """The attention kernel a dense pass of this workload launches: one CTA per
+    (sequence, head, 128-query tile) item for head_dim 64, and for head_dim 128
+    while the items fit on the SMs; else the persistent two-query-tile kernel."""
     if cfg["head_dim"] != 128:
-        return "attention_kernel"
+        return "attention_tc_kernel<64>"
     import torch
     items = -(-(cfg["prompt_len"] + cfg["gen_len"]) // 128) * cfg["n_heads"] * cfg["batch"]
     sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
-    return "attention_tc_kernel" if items <= sms else "attention_tc2_kernel"
+    return "attention_tc_kernel<128>" if items <= sms else "attention_tc2_kernel"
 
 
 def tiny_leg(reps: int = 5):

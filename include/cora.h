@@ -290,7 +290,10 @@ CORA_API int cora_session_disagreement(cora_session* s, cora_session* dense, int
 #define CORA_KIND_GATE 9           /* Eq. 1 combine + transfer rule + Eq. 2-4 */
 
 /* Runs one cora_denoise_step without the CUDA graph, with CUDA events around
- * every kernel launch, for profiling.  It is a real step (state advances).
+ * every kernel launch, for profiling.  It is a real step (state advances) and
+ * runs the pass the next cora_denoise_step would run (in a prefix-cache
+ * session: the block's dense first pass, or a pass over the rows from the
+ * active block on).
  *   capacity  size of kinds/ms (>= 4 + 7 * n_layers)
  *   kinds     host int32 [capacity] (out): CORA_KIND_* of each launch, in order
  *   ms        host float [capacity] (out): device time of each launch

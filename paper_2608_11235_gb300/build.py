@@ -21,8 +21,8 @@ OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libcora.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 
-SOURCES = ["runtime.cu", "gemm.cu", "gemm_skinny.cu", "lm_head.cu", "attention.cu", "attention_tc.cu",
-           "attention_tc2.cu", "gate.cu", "synth_norm.cu"]
+SOURCES = ["runtime.cu", "gemm.cu", "gemm_skinny.cu", "lm_head.cu", "attention_tc.cu", "attention_tc2.cu", "gate.cu",
+           "synth_norm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr", "-I", INCLUDE]

@@ -1,8 +1,9 @@
 // Bidirectional (non-causal) attention on the 5th-generation tensor cores,
-// head_dim 128.  Work item = (sequence, query head, 128-query tile).
-// attention_tc_kernel runs one item per CTA and serves launches whose items
-// fit on the SMs at once; launches with more items than SMs go to the
-// two-query-tile persistent kernel (attention_tc2.cu).  Keys and values
+// head_dim 128 or 64.  Work item = (sequence, query head, 128-query tile).
+// attention_tc_kernel runs one item per CTA and serves head_dim 64 launches
+// and head_dim 128 launches whose items fit on the SMs at once; head_dim 128
+// launches with more items than SMs go to the two-query-tile persistent
+// kernel (attention_tc2.cu).  Keys and values
 // stream through shared memory in 128-key tiles (TMA, double-buffered).
 //
 // Per key tile j:
@@ -36,9 +37,13 @@ namespace cora {
 namespace attn {
 constexpr int QT = 128;          // queries per CTA
 constexpr int KT = 128;          // keys per tile
-constexpr int HD = 128;          // head dim
-constexpr int OPND = QT * HD * 2;  // 32 KB: one 128 x 128 bf16 operand (two 16 KB swizzle columns)
-constexpr int SMEM = 7 * OPND + 1024 + 256;  // Q, K[2], V[2], P[2]
+constexpr int COL = 128 * 128;   // 16 KB: one 128-row x 64-element swizzle column of a bf16 operand
+// Shared memory for head dim hd: Q, K[2], V[2] of hd/64 columns each, P[2] of two columns (128 keys).
+template <int HD>
+struct Tile {
+  static constexpr int OPND = COL * (HD / 64);
+  static constexpr int SMEM = 5 * OPND + 4 * COL + 1024 + 256;
+};
 constexpr float kRescale = 8.0f; // log2 headroom before the reference max is raised
 }  // namespace attn
 
@@ -104,21 +109,24 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, const void*
 // One CTA per item (grid = query tiles x heads x sequences): used when the
 // items fit on the SMs at once.  (On 128 items at S = 512 it measured 12.6 us
 // against 13.5 us for a persistent one-tile-per-item variant, ncu, same command.)
+template <int HD>
 __global__ void __launch_bounds__(192, 1)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tmQKV, const __grid_constant__ CUtensorMap tmOut, int S,
                         int Hq, int Hkv, int q_start, int* err) {
   using namespace attn;
-  // idesc: M = 128, N = 128, bf16 x bf16 -> f32; PV reads B (V) MN-major.
+  constexpr int OPND = Tile<HD>::OPND;
+  constexpr int NC = HD / 64;  // swizzle columns of a Q / K / V tile
+  // idesc: QK M = 128, N = 128 (keys); PV M = 128, N = hd, B (V) MN-major; bf16 x bf16 -> f32.
   constexpr uint32_t IDESC_QK = idesc_bf16_f32(128, 128);
-  constexpr uint32_t IDESC_PV = idesc_bf16_f32(128, 128) | (1u << 16);
+  constexpr uint32_t IDESC_PV = idesc_bf16_f32(128, HD) | (1u << 16);
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
   uint8_t* sK[2] = {smem + OPND, smem + 2 * OPND};
   uint8_t* sV[2] = {smem + 3 * OPND, smem + 4 * OPND};
-  uint8_t* sP[2] = {smem + 5 * OPND, smem + 6 * OPND};
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 7 * OPND);
+  uint8_t* sP[2] = {smem + 5 * OPND, smem + 5 * OPND + 2 * COL};
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 5 * OPND + 4 * COL);
   uint64_t* qfull = bars + 0;
   uint64_t* kfull = bars + 1;    // [2] K_j landed
   uint64_t* vfull = bars + 3;    // [2] V_j landed
@@ -173,20 +181,17 @@ __global__ void __launch_bounds__(192, 1)
   if (warp == 0) {
     if (lane == 0) {
       mbar_arrive_expect_tx(qfull, OPND);
-      tma_load_2d(sQ, &tmQKV, qfull, qcol, row_base + q0);
-      tma_load_2d(sQ + OPND / 2, &tmQKV, qfull, qcol + 64, row_base + q0);
+      for (int c = 0; c < NC; ++c) tma_load_2d(sQ + c * COL, &tmQKV, qfull, qcol + c * 64, row_base + q0);
       for (int j = 0; j < n_kt; ++j) {
         const int s = j & 1;
         const uint32_t ph = ((j >> 1) & 1) ^ 1u;
         const int r = row_base + j * KT;
         if (!mbar_wait(&kempty[s], ph, abort_flag, err, CORA_DERR_TMA_WAIT)) break;
         mbar_arrive_expect_tx(&kfull[s], OPND);
-        tma_load_2d(sK[s], &tmQKV, &kfull[s], kcol, r);
-        tma_load_2d(sK[s] + OPND / 2, &tmQKV, &kfull[s], kcol + 64, r);
+        for (int c = 0; c < NC; ++c) tma_load_2d(sK[s] + c * COL, &tmQKV, &kfull[s], kcol + c * 64, r);
         if (!mbar_wait(&vempty[s], ph, abort_flag, err, CORA_DERR_TMA_WAIT)) break;
         mbar_arrive_expect_tx(&vfull[s], OPND);
-        tma_load_2d(sV[s], &tmQKV, &vfull[s], vcol, r);
-        tma_load_2d(sV[s] + OPND / 2, &tmQKV, &vfull[s], vcol + 64, r);
+        for (int c = 0; c < NC; ++c) tma_load_2d(sV[s] + c * COL, &tmQKV, &vfull[s], vcol + c * 64, r);
       }
     }
   } else if (warp == 1) {
@@ -204,9 +209,9 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
         for (int k = 0; k < KT / 16; ++k) {
           // A = P: K-major, keys contiguous, 64-key swizzle columns 16 KB apart.
-          const uint64_t a = sw128_kmajor_desc(p_addr + (k >> 2) * (OPND / 2) + (k & 3) * 32);
+          const uint64_t a = sw128_kmajor_desc(p_addr + (k >> 2) * COL + (k & 3) * 32);
           // B = V: rows are keys (K), 64-element hd blocks 16 KB apart (MN-major).
-          const uint64_t bd = sw128_mnmajor_desc(v_addr + k * 16 * 128, OPND / 2);
+          const uint64_t bd = sw128_mnmajor_desc(v_addr + k * 16 * 128, COL);
           umma_bf16(o_tmem, a, bd, IDESC_PV, (jj > 0 || k > 0) ? 1u : 0u);
         }
         umma_commit(&pdone[s]);
@@ -223,7 +228,7 @@ __global__ void __launch_bounds__(192, 1)
         const uint32_t d = tmem_base + s * 128;
 #pragma unroll
         for (int k = 0; k < HD / 16; ++k) {
-          const uint32_t off = (k >> 2) * (OPND / 2) + (k & 3) * 32;
+          const uint32_t off = (k >> 2) * COL + (k & 3) * 32;
           umma_bf16(d, sw128_kmajor_desc(q_addr + off), sw128_kmajor_desc(k_addr + off), IDESC_QK, k > 0);
         }
         umma_commit(&sfull[s]);
@@ -305,7 +310,7 @@ __global__ void __launch_bounds__(192, 1)
         }
         // keys c .. c+7 -> swizzle column c/64, 16-byte chunk (c%64)/8
         const int chunk = (c & 63) >> 3;
-        *reinterpret_cast<uint4*>(prow + (c >> 6) * (OPND / 2) + r * 128 + ((chunk ^ (r & 7)) << 4)) =
+        *reinterpret_cast<uint4*>(prow + (c >> 6) * COL + r * 128 + ((chunk ^ (r & 7)) << 4)) =
             make_uint4(pk[0], pk[1], pk[2], pk[3]);
       }
       l += (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
@@ -322,24 +327,28 @@ __global__ void __launch_bounds__(192, 1)
     }
     if (ok) {
       tc_fence_after();
-      uint32_t o[128];
-      tmem_ld128(o_lane, o);
       const float inv = 1.f / l;
       uint8_t* stg = sP[0];
+#pragma unroll 1
+      for (int c0 = 0; c0 < HD; c0 += 32) {
+        uint32_t o[32];
+        tmem_ld32w(o_lane + c0, o);
 #pragma unroll
-      for (int c = 0; c < HD; c += 8) {
-        const int chunk = (c & 63) >> 3;
-        *reinterpret_cast<uint4*>(stg + (c >> 6) * (OPND / 2) + r * 128 + ((chunk ^ (r & 7)) << 4)) = make_uint4(
-            pack_bf16x2(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
-            pack_bf16x2(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
-            pack_bf16x2(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
-            pack_bf16x2(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
+        for (int i = 0; i < 32; i += 8) {
+          const int c = c0 + i;
+          const int chunk = (c & 63) >> 3;
+          *reinterpret_cast<uint4*>(stg + (c >> 6) * COL + r * 128 + ((chunk ^ (r & 7)) << 4)) = make_uint4(
+              pack_bf16x2(__uint_as_float(o[i]) * inv, __uint_as_float(o[i + 1]) * inv),
+              pack_bf16x2(__uint_as_float(o[i + 2]) * inv, __uint_as_float(o[i + 3]) * inv),
+              pack_bf16x2(__uint_as_float(o[i + 4]) * inv, __uint_as_float(o[i + 5]) * inv),
+              pack_bf16x2(__uint_as_float(o[i + 6]) * inv, __uint_as_float(o[i + 7]) * inv));
+        }
       }
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) {
-        for (int c = 0; c < 2; ++c)
-          tma_store_3d(&tmOut, stg + c * (OPND / 2) + sub * 32 * 128, qcol + c * 64, qt * QT + sub * 32, b);
+        for (int c = 0; c < NC; ++c)
+          tma_store_3d(&tmOut, stg + c * COL + sub * 32 * 128, qcol + c * 64, qt * QT + sub * 32, b);
         asm volatile("cp.async.bulk.commit_group;" ::: "memory");
         asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
       }
@@ -363,23 +372,29 @@ __global__ void __launch_bounds__(192, 1)
 using namespace cora;
 
 cudaError_t attention_tc_prepare() {
-  return cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, attn::SMEM);
+  cudaError_t e = cudaFuncSetAttribute(attention_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       attn::Tile<128>::SMEM);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attention_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              attn::Tile<64>::SMEM);
 }
 
-cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
-                                int q_len, int* err, int num_sms, cudaStream_t st) {
+cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int hd,
+                                int q_start, int q_len, int* err, int num_sms, cudaStream_t st) {
   // Output map [B][q_len][Hq*hd] bf16, boxes of 32 rows x 64 columns (one
   // warp's rows, one 128-byte swizzle column).
   CUtensorMap tmOut;
-  if (!make_tmap_bf16_3d(&tmOut, out, static_cast<uint64_t>(Hq) * attn::HD, q_len, B,
-                         static_cast<uint64_t>(Hq) * attn::HD * 2, static_cast<uint64_t>(q_len) * Hq * attn::HD * 2,
-                         64, 32, 1))
+  if (!make_tmap_bf16_3d(&tmOut, out, static_cast<uint64_t>(Hq) * hd, q_len, B, static_cast<uint64_t>(Hq) * hd * 2,
+                         static_cast<uint64_t>(q_len) * Hq * hd * 2, 64, 32, 1))
     return cudaErrorInvalidValue;
   const int n_qt = (q_len + attn::QT - 1) / attn::QT;
   const int n_items = n_qt * Hq * B;
+  if (hd == 64)  // one CTA per item, in as many waves as it takes
+    return launch_pdl(attention_tc_kernel<64>, dim3(n_qt, Hq, B), dim3(192), attn::Tile<64>::SMEM, st, tmQKV, tmOut,
+                      S, Hq, Hkv, q_start, err);
   if (n_items <= num_sms)
-    return launch_pdl(attention_tc_kernel, dim3(n_qt, Hq, B), dim3(192), attn::SMEM, st, tmQKV, tmOut, S, Hq, Hkv,
-                      q_start, err);
+    return launch_pdl(attention_tc_kernel<128>, dim3(n_qt, Hq, B), dim3(192), attn::Tile<128>::SMEM, st, tmQKV,
+                      tmOut, S, Hq, Hkv, q_start, err);
   // More items than SMs: two query tiles per CTA (attention_tc2.cu).
   return launch_attention_tc2(tmQKV, out, B, S, Hq, Hkv, q_start, q_len, err, num_sms, st);
 }

@@ -201,25 +201,22 @@ cudaError_t launch_lm_head_top1(const CUtensorMap& tmW, const CUtensorMap& tmX, 
 // outside stream capture).
 cudaError_t gemm_prepare();
 cudaError_t lm_head_prepare();
-cudaError_t attention_prepare();
 cudaError_t attention_tc_prepare();
 cudaError_t attention_tc2_prepare();
 // Two query tiles per CTA, persistent over (sequence, head, query-tile pair)
 // items; out bf16 [B][q_len][Hq*128] written directly.
 cudaError_t launch_attention_tc2(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
                                  int q_len, int* err, int num_sms, cudaStream_t st);
-// tcgen05 attention for head_dim 128; tmQKV: bf16 [B*S, (Hq+2Hkv)*128], box 128 rows x 64 cols.
-// Items = ceil(q_len/128) * Hq * B: one CTA per item when they fit on the SMs,
-// else the two-query-tile persistent kernel (launch_attention_tc2).
-cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int q_start,
-                                int q_len, int* err, int num_sms, cudaStream_t st);
+// tcgen05 attention, head_dim hd in {64, 128}; tmQKV: bf16 [B*S, (Hq+2Hkv)*hd], box 128 rows x 64 cols.
+// Queries q_start .. q_start + q_len - 1 of every sequence against all S keys;
+// out holds q_len rows per sequence ((0, S): the dense pass).  Items =
+// ceil(q_len/128) * Hq * B: one CTA per item (hd 64; hd 128 when they fit on
+// the SMs), else the two-query-tile persistent kernel (launch_attention_tc2).
+cudaError_t launch_attention_tc(const CUtensorMap& tmQKV, uint16_t* out, int B, int S, int Hq, int Hkv, int hd,
+                                int q_start, int q_len, int* err, int num_sms, cudaStream_t st);
 
 void launch_session_init(int32_t* tokens, const int32_t* prompt, uint8_t* state, int32_t* persist, int32_t* prev,
                          int32_t* ctrl, int32_t* status, int B, int P, int S, int G, int BL, int mask_id,
                          cudaStream_t st);
 
-// Attention.
-// Queries q_start .. q_start + q_len - 1 of every sequence against all S keys;
-// out holds q_len rows per sequence.  (0, S): the dense pass.
-void launch_attention(const uint16_t* qkv, uint16_t* out, int B, int S, int Hq, int Hkv, int hd, int q_start,
-                      int q_len, cudaStream_t st);
+

@@ -176,7 +176,6 @@ static int kernels_prepare() {
   if (!dc->prepared) {
     CK(gemm_prepare());
     CK(lm_head_prepare());
-    CK(attention_prepare());
     CK(attention_tc_prepare());
     CK(attention_tc2_prepare());
     dc->prepared = true;
@@ -520,12 +519,8 @@ static int enqueue_step(cora_session* s, LaunchRecorder* rec = nullptr,
     const CUtensorMap& tmo = packed ? s->tmo_qkv3_l[l] : cache ? s->tmo_qkv_l[l] : s->tmo_qkv;
     CK(launch_gemm(s->tm_xn, m->tm_qkv[l], tmo, M, m->n_qkv, d, e1, s->gemm_ws, err, m->num_sms, st));
     REC(CORA_KIND_GEMM_QKV);
-    if (c.head_dim == 128) {
-      CK(launch_attention_tc(cache ? s->tm_qkv_in_l[l] : s->tm_qkv_in, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads,
-                             lo, Ls, err, m->num_sms, st));
-    } else {
-      launch_attention(qkv, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads, c.head_dim, lo, Ls, st);
-    }
+    CK(launch_attention_tc(cache ? s->tm_qkv_in_l[l] : s->tm_qkv_in, s->attn, s->B, s->S, c.n_heads, c.n_kv_heads,
+                           c.head_dim, lo, Ls, err, m->num_sms, st));
     REC(CORA_KIND_ATTENTION);
     GemmEpilogue e2{s->h, d, CORA_EPI_RESID_F32, nullptr, 0, 0, 0, 1};
     e2.a_ptr = s->attn;
@@ -925,9 +920,13 @@ extern "C" int cora_session_profile_step(cora_session* s, int32_t capacity, int3
   REQUIRE(capacity >= need, "cora_session_profile_step: capacity %d < %d launches", capacity, need);
   CK(cudaStreamSynchronize(s->stream));
   LaunchRecorder rec;
-  int rc = enqueue_step(s, &rec);
+  // The pass the next cora_denoise_step would run: in a prefix-cache session
+  // a later pass of the current block covers the rows from it on.
+  const int cached_block = (!s->cgraph.empty() && !(s->next_info & 1)) ? (s->next_info >> 1) : -1;
+  int rc = enqueue_step(s, &rec, nullptr, cached_block);
   if (rc) return rc;
   CK(cudaStreamSynchronize(s->stream));
+  if (!s->cgraph.empty()) s->next_info = s->status_h[3];
   s->batched_passes += 1;
   const int n = static_cast<int>(rec.kinds.size());
   for (int i = 0; i < n; ++i) {
@@ -1147,18 +1146,14 @@ extern "C" int cora_op_attention_rows(const uint16_t* qkv, uint16_t* out, int32_
   REQUIRE(aligned16(qkv) && aligned16(out), "cora_op_attention: pointers must be 16-byte aligned");
   int rc = kernels_prepare();
   if (rc) return rc;
-  if (hd == 128) {
-    DeviceCtx* dc = nullptr;
-    if ((rc = device_ctx(&dc))) return rc;
-    CUtensorMap tq;
-    const size_t cols = size_t(Hq + 2 * Hkv) * hd;
-    if (!make_tmap_bf16_2d(&tq, qkv, size_t(B) * S, cols, cols * 2, 128, 64))
-      return fail(CORA_ECUDA, "cora_op_attention: tensor map encoding failed");
-    CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, q_start, q_len, dc->err, dc->num_sms,
-                           static_cast<cudaStream_t>(stream)));
-  } else {
-    launch_attention(qkv, out, B, S, Hq, Hkv, hd, q_start, q_len, static_cast<cudaStream_t>(stream));
-  }
+  DeviceCtx* dc = nullptr;
+  if ((rc = device_ctx(&dc))) return rc;
+  CUtensorMap tq;
+  const size_t cols = size_t(Hq + 2 * Hkv) * hd;
+  if (!make_tmap_bf16_2d(&tq, qkv, size_t(B) * S, cols, cols * 2, 128, 64))
+    return fail(CORA_ECUDA, "cora_op_attention: tensor map encoding failed");
+  CK(launch_attention_tc(tq, out, B, S, Hq, Hkv, hd, q_start, q_len, dc->err, dc->num_sms,
+                         static_cast<cudaStream_t>(stream)));
   CK(cudaGetLastError());
   return CORA_OK;
 }

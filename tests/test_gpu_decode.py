@@ -434,6 +434,31 @@ def test_prefix_cache_matches_oracle_hd128():
         cora.cora_model_destroy(m)
 
 
+def test_profile_step_runs_the_cached_pass(tiny):
+    """cora_session_profile_step runs the pass the next step would run: on a
+    prefix-cache session after a block's dense first pass, the pass over the
+    rows from the block on.  Same pre-step state through the profiled eager
+    pass and through cora_denoise_step: identical Eq. 1 outputs and state."""
+    m, _, prompt = tiny
+    s = cora.cora_session_create(m, 1, prompt[:1], P, G, BL, T, TAU, K,
+                                 options=cora.decode_options(cache=cora.CACHE_PREFIX))
+    try:
+        cora.cora_denoise_step(s, 0, 0)                       # block 0's dense first pass
+        st = cora.cora_session_read(s, 1, P + G, G, BL)
+        prof = cora.cora_session_profile_step(s, CFG["n_layers"])
+        assert len(prof) == 4 + 7 * CFG["n_layers"]
+        a = cora.cora_session_read(s, 1, P + G, G, BL)
+        cora.cora_session_write(s, tokens=st["tokens"], state=st["state"], persist=st["persist"], prev=st["prev"],
+                                ctrl=st["ctrl"])
+        cora.cora_denoise_step(s, 0, 1)                       # the same cached pass through the graph
+        b = cora.cora_session_read(s, 1, P + G, G, BL)
+        for key in ("conf", "argmax", "tokens", "state", "persist", "prev", "unmask", "accept"):
+            assert np.array_equal(a[key], b[key]), key
+        assert a["ctrl"][0, :2].tolist() == b["ctrl"][0, :2].tolist()
+    finally:
+        cora.cora_session_destroy(s)
+
+
 def test_prefix_cache_batch_moves_blocks_together(sharp):
     """Prefix-cache sessions move a batch's sequences to the next block
     together: unfinished sequences always share the block index, a sequence
