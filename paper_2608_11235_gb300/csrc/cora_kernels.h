@@ -129,6 +129,12 @@ struct GemmEpilogue {
   int splits;
   int split_skew;
   int split_pair;  // 1: two k-pieces per tile, each finalising half of the columns
+  // Set by launch_gemm: whole tiles per unit (CTA pair) run in data-parallel
+  // waves after the stream-K tiles, the row blocks per group of the tile
+  // numbering (1: M-slowest), and the units sharing the stream-K tiles.
+  int dp_waves;
+  int raster_group;
+  int sk_units;
   // ROPE epilogue on packed prefix-cache rows: row r is position
   // rope_pos0 + r % seq of sequence r / seq; with out3d, C is a 3-D map
   // [sequence][position][column] and row r is stored at that position.

@@ -26,6 +26,17 @@
 // weight tile (B) for different row blocks run concurrently and share it
 // through L2.  Two TMEM accumulators (2 * BN columns) let the epilogue of one
 // segment overlap the MMAs of the next.
+//
+// Many tiles (the 2-CTA kernel, more than two row blocks, at least one tile
+// per unit): stream-K covers only the remainder, tiles mod units, and the
+// rest run as whole tiles in data-parallel waves (unit c takes tile
+// sk + w P + c in wave w), with tiles numbered in groups of row blocks, row
+// block fastest (see tile_coords).  A contiguous range per unit over
+// thousands of tiles would put the units' concurrent tiles all over the tile
+// grid, every one on its own weight tile, each unit at its own k-offset; a
+// wave of consecutive tiles covers a few row blocks and weight tiles, every
+// unit at the same k-block, so each k-slice of a shared operand comes from
+// DRAM once and from L2 for the other units.
 #include <math.h>
 
 #include <algorithm>
@@ -59,7 +70,10 @@ struct GemmCfg {
 // piece skew shorter, so the other pieces' partials are written while the
 // finisher is still issuing MMAs instead of after.
 struct WorkSplit {
-  int G, W, KB, S, skew;
+  int G, W, KB, S, skew;  // G: the units sharing the stream-K tiles (the first W / KB)
+  // Whole tiles each of the P units runs after its stream-K range: unit c
+  // runs tile W / KB + w P + c in wave w.
+  int dp_waves, P;
   __device__ int start(int c) const {
     if (skew > 0) {
       const int t = c / S, s = c - t * S;
@@ -72,28 +86,36 @@ struct WorkSplit {
 // A CTA's iteration range as segments (tile, kb0, kb1), visited in the order
 // (1) its first segment (a contributor when it starts mid-tile), (2) its
 // last segment (a split tile it finishes when it ends mid-tile), (3) the
-// whole tiles in between.  Putting both split segments first lets their
-// hand-off and fix-up overlap the MMAs of the whole tiles.
+// whole tiles in between, (4) its data-parallel tiles.  Putting both split
+// segments first lets their hand-off and fix-up overlap the MMAs of the
+// whole tiles.
 struct SegIter {
-  int it0, it1, kb_per_tile, t_first, t_last, idx;
+  int it0, it1, kb_per_tile, t_first, t_last, idx, n_sk, dp_t0, dp_stride, dp_n;
   __device__ SegIter(int c, const WorkSplit& ws)
-      : it0(ws.start(c)), it1(ws.start(c + 1)), kb_per_tile(ws.KB), idx(0) {
+      : it0(c < ws.G ? ws.start(c) : ws.W), it1(c < ws.G ? ws.start(c + 1) : ws.W), kb_per_tile(ws.KB), idx(0) {
     t_first = it0 / ws.KB;
     t_last = it1 > it0 ? (it1 - 1) / ws.KB : t_first - 1;
+    n_sk = it1 <= it0 ? 0 : (t_first == t_last ? 1 : 2 + (t_last - t_first - 1));
+    dp_t0 = ws.W / ws.KB + c;
+    dp_stride = ws.P;
+    dp_n = ws.dp_waves;
   }
   __device__ bool next(int& t, int& kb0, int& kb1) {
-    if (it1 <= it0) return false;
     const int KB = kb_per_tile;
-    if (t_first == t_last) {  // the whole range lies in one tile
-      if (idx++ > 0) return false;
+    if (idx >= n_sk) {  // data-parallel whole tiles
+      const int w = idx - n_sk;
+      if (w >= dp_n) return false;
+      t = dp_t0 + w * dp_stride;
+      kb0 = 0;
+      kb1 = KB;
+      ++idx;
+      return true;
+    }
+    if (t_first == t_last) {  // the whole stream-K range lies in one tile
       t = t_first;
       kb0 = it0 - t * KB;
       kb1 = it1 - t * KB;
-      return true;
-    }
-    const int n_mid = t_last - t_first - 1;
-    if (idx >= 2 + n_mid) return false;
-    if (idx == 0) {
+    } else if (idx == 0) {
       t = t_first;
       kb0 = it0 - t * KB;
       kb1 = KB;
@@ -110,12 +132,20 @@ struct SegIter {
     return true;
   }
   // True once the segment just returned is the last one this CTA visits.
-  __device__ bool finished() const {
-    if (it1 <= it0) return true;
-    if (t_first == t_last) return idx > 0;
-    return idx >= 2 + (t_last - t_first - 1);
-  }
+  __device__ bool finished() const { return idx >= n_sk + dp_n; }
 };
+
+// Row block and column block of tile t: tiles are numbered in groups of
+// `group` row blocks (the last group may be smaller), row block fastest
+// within a group, so consecutive tiles share weight tiles (B) and the group's
+// row blocks (A) stay in L2 while its columns are walked.  group = 1: M-slowest.
+__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group, int& mb, int& nb) {
+  const int per_group = group * num_n;
+  const int g = t / per_group, r = t - g * per_group;
+  const int gm = min(group, num_m - g * group);
+  mb = g * group + r % gm;
+  nb = r / gm;
+}
 
 // Walks a CTA's (tile, k-block) sequence in the order the producer loads it.
 struct KbCursor {
@@ -522,7 +552,7 @@ __global__ void __launch_bounds__(192, 1)
   const int KB = K / kBK;
   const int W = num_tiles * KB;
   const int G = gridDim.x;
-  const WorkSplit wsplit{G, W, KB, ep.splits, ep.split_skew};
+  const WorkSplit wsplit{G, W, KB, ep.splits, ep.split_skew, 0, G};
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -854,10 +884,12 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
   const int pair = blockIdx.x >> 1;
   const int G = gridDim.x >> 1;
   const int num_n = N / BN;
-  const int num_tiles = ((M + 255) / 256) * num_n;
+  const int num_m = (M + 255) / 256;
+  const int num_tiles = num_m * num_n;
   const int KB = K / kBK;
-  const int W = num_tiles * KB;
-  const WorkSplit wsplit{G, W, KB, ep.splits, ep.split_skew};
+  const int W = (num_tiles - ep.dp_waves * G) * KB;  // the stream-K tiles' iterations
+  const WorkSplit wsplit{ep.sk_units, W, KB, ep.splits, ep.split_skew, ep.dp_waves, G};
+  const int group = ep.raster_group;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -899,8 +931,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
     for (KbCursor cur(pair, wsplit); n_pre < STAGES && cur.valid; ++n_pre, cur.advance()) {
       uint8_t* sa = smem + n_pre * Cfg::STAGE_BYTES;
       if (leader) mbar_arrive_expect_tx(&full[n_pre], 2 * Cfg::STAGE_BYTES);
+      int pmb, pnb;
+      tile_coords(cur.t, num_m, num_n, group, pmb, pnb);
       tma_load_2d_pair(sa + Cfg::A_BYTES, &tmB, mapa_shared(smem_u32(&full[n_pre]), 0), cur.kb * kBK,
-                       (cur.t % num_n) * BN + b_row);
+                       pnb * BN + b_row);
     }
   }
   pdl_wait();
@@ -912,7 +946,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
       SegIter seg(pair, wsplit);
       int t, kb0, kb1;
       while (seg.next(t, kb0, kb1)) {
-        const int mb = t / num_n, nb = t - mb * num_n;
+        int mb, nb;
+        tile_coords(t, num_m, num_n, group, mb, nb);
         for (int kb = kb0; kb < kb1; ++kb) {
           uint8_t* sa = smem + stage * Cfg::STAGE_BYTES;
           const uint32_t lead_full = mapa_shared(smem_u32(&full[stage]), 0);
@@ -990,7 +1025,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
       const bool ok = mbar_wait(&tfull[acc], acc_phase, abort_flag, err, CORA_DERR_EPI_WAIT);
       if (named_bar_or(1, 128, !ok)) break;
       tc_fence_after();
-      const int mb = t / num_n, nb = t - mb * num_n;
+      int mb, nb;
+      tile_coords(t, num_m, num_n, group, mb, nb);
       const uint32_t tacc = tmem_base + (static_cast<uint32_t>(sub * 32) << 16) + acc * BN;
       const int row0 = mb * 256 + static_cast<int>(rank) * 128 + sub * 32;
       if (ep.split_pair) {
@@ -1052,7 +1088,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(192, 1)
         const int last_it = t * KB + KB - 1;
         c_first = pair + 1;
         c_last = c_first;
-        while (c_last + 1 < G && wsplit.start(c_last + 1) <= last_it) ++c_last;
+        while (c_last + 1 < wsplit.G && wsplit.start(c_last + 1) <= last_it) ++c_last;
         const int n_c = c_last - c_first + 1;
         const bool bulk = seg.finished() && n_c * kBM * BN * 4 <= STAGES * Cfg::STAGE_BYTES;
         bool fok = true;
@@ -1172,6 +1208,9 @@ static int gemm_grid(int M, int N, int K, int bn, int num_sms, GemmEpilogue& ep)
   ep.splits = 0;
   ep.split_skew = 0;
   ep.split_pair = 0;
+  ep.dp_waves = 0;
+  ep.raster_group = 1;
+  ep.sk_units = 0;  // set below to the grid
   if (2 * tiles <= num_sms) {
     // Few tiles: split every tile into the same number of k-ranges (at most
     // 4), so each CTA holds one piece and every finisher has its operand
@@ -1189,13 +1228,15 @@ static int gemm_grid(int M, int N, int K, int bn, int num_sms, GemmEpilogue& ep)
       ep.splits = splits;
       ep.split_skew = skew;
     }
+    ep.sk_units = tiles * splits;
     return tiles * splits;
   }
   long long g = num_sms;
   const long long max_by_share = W / ((KB + 3) / 4);
   if (g > max_by_share) g = max_by_share;
   if (g > W) g = W;
-  return g < 1 ? 1 : static_cast<int>(g);
+  ep.sk_units = g < 1 ? 1 : static_cast<int>(g);
+  return ep.sk_units;
 }
 
 template <int BN>
@@ -1209,10 +1250,32 @@ static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB
                     err);
 }
 
+// Row blocks per group of the tile numbering when a GEMM runs data-parallel
+// waves: a wave of 76 pair-tiles then covers 8 row blocks and ~10 weight
+// tiles.
+constexpr int kRasterGroup = 8;
+
 // Pairs for the 2-CTA kernel: the 1-CTA rule applied to 256 x 256 pair-tiles
-// and half the SMs.
+// and half the SMs.  With more than two row blocks and at least one tile per
+// pair, the tiles run as data-parallel waves over the grouped numbering
+// (every pair starts each wave's tile at k-block 0, so the pairs sharing a row
+// block or a weight tile read each k-slice of it at about the same time and
+// L2 serves all but the first), and only the remainder (tiles mod pairs) is
+// split stream-K, first, over as many pairs as give each at least a quarter
+// of a tile.  (With one or two row blocks the M-slowest stream-K order already
+// runs the pairs that share a weight tile side by side: pair p and p + G/2.)
 static int gemm2_pairs(int M, int N, int K, int num_sms, GemmEpilogue& ep) {
-  return gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2, ep);
+  const int pairs = gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2, ep);
+  const int num_m = (M + 255) / 256;
+  const int tiles = num_m * (N / 256);
+  if (ep.splits == 0 && num_m > 2 && tiles >= pairs) {
+    const int KB = K / kBK;
+    const int rem = tiles % pairs;
+    ep.dp_waves = tiles / pairs;
+    ep.raster_group = kRasterGroup;
+    ep.sk_units = rem == 0 ? pairs : std::min(pairs, std::max(1, rem * KB / ((KB + 3) / 4)));
+  }
+  return pairs;
 }
 
 cudaError_t launch_wait_check(int which, const int* flag, int* err, cudaStream_t st) {

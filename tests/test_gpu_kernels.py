@@ -88,7 +88,9 @@ def run_gemm(A, Bm, M, N, K, epi, out_cols, out_dtype=torch.int16, C0=None, **kw
 @pytest.mark.parametrize("M,N,K", [(300, 512, 320), (128, 384, 64), (2048, 4096, 256), (256, 256, 4096),
                                    (96, 768, 256), (1, 256, 128), (512, 4096, 4096), (512, 12288, 1024),
                                    (96, 768, 2048), (128, 16384, 512),
-                                   (64, 12288, 1024), (16, 4096, 4096), (5, 384, 640)])   # few-row kernel
+                                   (64, 12288, 1024), (16, 4096, 4096), (5, 384, 640),    # few-row kernel
+                                   (2048, 12288, 256),   # 384 pair-tiles: stream-K + 4 data-parallel waves
+                                   (1800, 10240, 192)])  # 320 pair-tiles, ragged last row block, 3 waves
 def test_gemm_store(M, N, K):
     A = bits(2, 10, (M, K), 1.0)
     Bm = bits(2, 11, (N, K), 1.0 / math.sqrt(K))
@@ -97,7 +99,8 @@ def test_gemm_store(M, N, K):
 
 
 @pytest.mark.parametrize("M,N,K", [(512, 4096, 4096),    # 32 pair-tiles: two skewed k-splits each
-                                   (512, 12288, 4096)])  # 96 pair-tiles over the SM pairs: stream-K
+                                   (512, 12288, 4096),   # 96 pair-tiles over the SM pairs: stream-K
+                                   (2048, 12288, 1024)])  # 384 pair-tiles: stream-K + data-parallel waves
 def test_gemm_split_tiles_are_deterministic(M, N, K):
     A = bits(2, 20, (M, K), 1.0)
     Bm = bits(2, 21, (N, K), 1.0 / math.sqrt(K))
@@ -107,7 +110,8 @@ def test_gemm_split_tiles_are_deterministic(M, N, K):
 
 
 @pytest.mark.parametrize("M,N,K", [(300, 512, 320), (130, 256, 1024), (512, 4096, 12288), (100, 16384, 512),
-                                   (40, 4096, 12288), (64, 16384, 512)])
+                                   (40, 4096, 12288), (64, 16384, 512),
+                                   (1536, 8192, 512)])  # 192 pair-tiles: stream-K + one data-parallel wave
 def test_gemm_residual(M, N, K):
     A = bits(3, 10, (M, K), 1.0)
     Bm = bits(3, 11, (N, K), 1.0 / math.sqrt(K))
@@ -117,7 +121,8 @@ def test_gemm_residual(M, N, K):
     assert np.abs(Ct.cpu().numpy() - ref).max() <= 1e-5 * np.abs(ref).max() + 1e-6
 
 
-@pytest.mark.parametrize("M,F,K", [(300, 256, 256), (96, 768, 256), (48, 4096, 4096), (7, 768, 256)])
+@pytest.mark.parametrize("M,F,K", [(300, 256, 256), (96, 768, 256), (48, 4096, 4096), (7, 768, 256),
+                                   (1100, 10240, 128)])  # 400 pair-tiles, ragged: stream-K + 4 waves
 def test_gemm_swiglu(M, F, K):
     A = bits(4, 10, (M, K), 1.0)
     g = bits(4, 11, (F, K), 1.0 / math.sqrt(K))
