@@ -8,6 +8,7 @@ residual gate with block termination) until every sequence has finished.
 Metric: generated tokens/s = batch * gen_len * steps / device time.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl cora|reference]
+  python bench.py --gemm-shapes-only FILTER   # the GEMM beside cuBLAS at the projection shapes
 
 Default workload: LLaDA-8B-shaped bidirectional Transformer (32 layers,
 d 4096, 32 heads x 128, SwiGLU 12288, vocab 126464), random-init bf16
@@ -47,8 +48,12 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # changed, and for workloads without a capture.
 NCU_TRAFFIC = {
     # gemm_tc2_kernel, mean of the QKV / O / gate-up / down launches (read + write):
-    # (124.4 + 46.3 + 245.1 + 125.6) MB / 4
-    ("gemm", "d8e0704d8d40", "llada8b-shape-256+256"): 135_355_000,
+    # (125.2 + 46.3 + 245.6 + 125.9) MB / 4
+    ("gemm", "9840a7e7c917", "llada8b-shape-256+256"): 135_742_528,
+    # (95.3 + 113.8 + 699.2 + 679.7) MB / 4
+    ("gemm", "9840a7e7c917", "dream7b-shape-256+512-b4"): 397_012_736,
+    # (1049.4 + 631.8 + 1667.1 + 1855.9) MB / 4
+    ("gemm", "9840a7e7c917", "llada8b-shape-512+1024-b8"): 1_301_025_792,
 }
 
 
@@ -377,6 +382,78 @@ def attention_shapes(peaks, reps: int = 5):
     return out
 
 
+def gemm_shapes(peaks, only: str = "", reps: int = 20, warmup: int = 3):
+    """The 2-SM GEMM alone at the four projection shapes of each 8B-class
+    workload's dense pass (M = batch x canvas rows), beside cuBLAS (torch.matmul,
+    bf16 out) on the same operands.  Epilogues as in the pass (residual fp32
+    add, SwiGLU), except QKV, timed with the plain bf16 store (the RoPE
+    epilogue needs a per-call table transpose).  CUDA events around `reps`
+    back-to-back launches on the same seeded operands, both sides alike;
+    `only` keeps the entries whose "workload/projection" name contains it."""
+    import torch
+
+    from paper_2608_11235_gb300 import configs, cora, synth
+
+    peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    out = {}
+    for name in ("llada8b-shape-256+256", "dream7b-shape-256+512-b4", "llada8b-shape-512+1024-b8"):
+        c = configs.PRESETS[name]
+        M = c["batch"] * (c["prompt_len"] + c["gen_len"])
+        d, hd = c["d_model"], c["head_dim"]
+        f = (c["ffn"] + 127) // 128 * 128
+        projs = (("qkv", (c["n_heads"] + 2 * c["n_kv_heads"]) * hd, d, cora.EPI_STORE_BF16),
+                 ("o", d, c["n_heads"] * hd, cora.EPI_RESID_F32),
+                 ("gate_up", 2 * f, d, cora.EPI_SWIGLU),
+                 ("down", d, f, cora.EPI_RESID_F32))
+        for proj, N, K, epi in projs:
+            key = f"{name}/{proj}"
+            if only and only not in key:
+                continue
+            A = torch.empty(M * K, dtype=torch.int16, device="cuda")
+            Bw = torch.empty(N * K, dtype=torch.int16, device="cuda")
+            cora.cora_synth_normal_bf16(A, M * K, synth.stream_key(31, 1), 0, float(synth.normal_scale_f32(1.0)))
+            cora.cora_synth_normal_bf16(Bw, N * K, synth.stream_key(31, 2), 0,
+                                        float(synth.normal_scale_f32(K ** -0.5)))
+            if epi == cora.EPI_RESID_F32:
+                C, ldc = torch.zeros(M, N, dtype=torch.float32, device="cuda"), N
+            elif epi == cora.EPI_SWIGLU:
+                C, ldc = torch.zeros(M, N // 2, dtype=torch.int16, device="cuda"), N // 2
+            else:
+                C, ldc = torch.zeros(M, N, dtype=torch.int16, device="cuda"), N
+
+            def ours():
+                cora.cora_op_gemm(A, Bw, C, M, N, K, ldc, epi)
+
+            At, Bt = A.view(torch.bfloat16).view(M, K), Bw.view(torch.bfloat16).view(N, K)
+            D = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+
+            def cublas():
+                torch.matmul(At, Bt.t(), out=D)
+
+            row = {"M": M, "N": N, "K": K, "epilogue": {0: "bf16 store", 1: "fp32 residual add", 2: "SwiGLU"}[epi]}
+            for tag, fn in (("ours", ours), ("cublas", cublas)):
+                for _ in range(warmup):
+                    fn()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                e0.record()
+                for _ in range(reps):
+                    fn()
+                e1.record()
+                e1.synchronize()
+                ms = e0.elapsed_time(e1) / reps
+                row[f"{tag}_us"] = round(ms * 1e3, 1)
+                row[f"{tag}_tflops"] = round(2.0 * M * N * K / (ms * 1e-3) / 1e12, 1)
+            row["ours_frac"] = round(row["ours_tflops"] / peak, 4)
+            row["vs_cublas"] = round(row["cublas_us"] / row["ours_us"], 3)
+            out[key] = row
+            del A, Bw, C, D
+            torch.cuda.empty_cache()
+    out["peak"] = peak
+    out["peak_source"] = "bf16 burst (kernels timed alone)"
+    return out
+
+
 def profile_pass(cora, s, cfg, prompt_dev):
     """Per-launch device times of the first pass of a decode, two eager runs
     (CUDA events around every launch on the session's stream), the smaller
@@ -634,6 +711,7 @@ def run_cora(args, cfg, ws, rank, local):
         peaks, with_oracle=(rank == 0 and ws == 1 and not args.no_cpu_baseline))
     tiny = None if args.no_variant else tiny_leg()
     attn_shapes = None if args.no_variant else attention_shapes(peaks)
+    gemm_cmp = None if args.no_variant else gemm_shapes(peaks)
 
     value = ws * B * G * args.steps / (ms * 1e-3)
     # embed, final norm, LM head, gate + per layer 2 RMSNorms, 4 GEMMs, attention; the device
@@ -667,6 +745,7 @@ def run_cora(args, cfg, ws, rank, local):
         "gate_isolation": gate_iso,
         "tiny": tiny,
         "attention_shapes": attn_shapes,
+        "gemm_shapes": gemm_cmp,
         "workloads": workloads,
     }
     return result, float(per_seq_passes.mean())
@@ -684,7 +763,16 @@ def main():
     ap.add_argument("--no-workloads", action="store_true",
                     help="skip the Dream-shaped and 512+1024 x 8 decodes (about four minutes)")
     ap.add_argument("--layers", type=int, default=0, help="override n_layers (same per-launch shapes)")
+    ap.add_argument("--gemm-shapes-only", default=None, metavar="FILTER",
+                    help="time only the GEMM-vs-cuBLAS shapes whose workload/projection name contains FILTER "
+                         "('' = all), print them as JSON and exit")
+    ap.add_argument("--gemm-reps", type=int, default=20)
     args = ap.parse_args()
+    if args.gemm_shapes_only is not None:
+        peaks, _ = load_peaks()
+        print(json.dumps(gemm_shapes(peaks, args.gemm_shapes_only, reps=args.gemm_reps,
+                                     warmup=min(args.warmup, 3))))
+        return
     from paper_2608_11235_gb300 import configs
     cfg = dict(configs.PRESETS[args.workload])
     if args.layers:

@@ -1262,8 +1262,11 @@ constexpr int kRasterGroup = 8;
 // block or a weight tile read each k-slice of it at about the same time and
 // L2 serves all but the first), and only the remainder (tiles mod pairs) is
 // split stream-K, first, over as many pairs as give each at least a quarter
-// of a tile.  (With one or two row blocks the M-slowest stream-K order already
-// runs the pairs that share a weight tile side by side: pair p and p + G/2.)
+// of a tile; the split tiles' hand-offs and fix-ups then run while the pair's
+// whole tiles are on the tensor cores.  With one or two row blocks the
+// M-slowest stream-K order already runs the pairs that share a weight tile
+// side by side (pair p and p + G/2), and there are too few whole tiles per
+// pair to hide a fix-up of up to four partials behind (measured slower).
 static int gemm2_pairs(int M, int N, int K, int num_sms, GemmEpilogue& ep) {
   const int pairs = gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2, ep);
   const int num_m = (M + 255) / 256;
