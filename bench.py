@@ -714,9 +714,10 @@ def run_cora(args, cfg, ws, rank, local):
     gemm_cmp = None if args.no_variant else gemm_shapes(peaks)
 
     value = ws * B * G * args.steps / (ms * 1e-3)
-    # embed, final norm, LM head, gate + per layer 2 RMSNorms, 4 GEMMs, attention; the device
-    # loop adds the kernel that counts the pass and sets the WHILE condition
-    launches_per_pass = 4 + 7 * cfg["n_layers"] + (1 if device_loop[0] else 0)
+    # the launches of one pass as the eager profile recorded them (embed, final norm, LM head,
+    # gate; per layer 4 GEMMs and attention, plus the RMSNorms not carried by a residual GEMM);
+    # the device loop adds the kernel that counts the pass and sets the WHILE condition
+    launches_per_pass = sum(k["launches_per_pass"] for k in kernels.values()) + (1 if device_loop[0] else 0)
     result = {
         "metric": "generated tokens/s (LLaDA-8B shape, gen 256)",
         "value": round(value, 3), "unit": "tokens/s", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,

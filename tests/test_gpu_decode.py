@@ -103,6 +103,44 @@ def test_replay_parity_every_step(tiny):
     print(f"replayed {len(tr.steps)} steps, {robust_steps} with flip-proof decisions, max|dc| = {max_dc:.2e}")
 
 
+def test_batched_replay_on_the_2sm_gemm(tiny):
+    """Three sequences at once: 3 x 96 = 288 rows, so every projection runs
+    on the 2-CTA GEMM (the single-sequence replays use the 1-CTA and few-row
+    kernels).  Step i of every sequence's oracle trace is replayed in one
+    batched step, each sequence at its own block and step: Eq. 1 within 2e-2,
+    argmax equal above the margin, the gate's rule on the GPU's own outputs."""
+    m, w, prompt = tiny
+    B = 3
+    trs = [O.generate(CFG, w, prompt[b], G, BL, T, TAU, K, record=True) for b in range(B)]
+    s = cora.cora_session_create(m, B, prompt, P, G, BL, T, TAU, K)
+    try:
+        n = min(12, *(len(tr.steps) for tr in trs))
+        max_dc = 0.0
+        for i in range(n):
+            sts = [tr.steps[i] for tr in trs]
+            ctrl = np.array([[st["block"], st["step"], st["passes_before"], 0] for st in sts], np.int32)
+            cora.cora_session_write(s, tokens=np.stack([st["canvas"] for st in sts]),
+                                    state=np.stack([st["gen_state"] for st in sts]),
+                                    persist=np.stack([st["before"].persist for st in sts]),
+                                    prev=np.stack([st["before"].prev for st in sts]), ctrl=ctrl)
+            cora.cora_denoise_step(s)
+            out = cora.cora_session_read(s, B, P + G, G, BL)
+            for b, st in enumerate(sts):
+                c, a = out["conf"][b], out["argmax"][b]
+                dc = np.abs(c - st["conf"])
+                max_dc = max(max_dc, float(dc.max()))
+                assert dc.max() <= 2e-2, (b, i, dc.max())
+                sel = O.top2_margin(st["logits"]) > 2e-2
+                assert np.array_equal(a[sel], st["x_hat"][sel]), (b, i)
+                k = O.transfer_schedule(BL, T)[st["step"]]
+                b0 = st["before"]
+                assert rule_holds(b0.state, b0.persist, b0.prev, c, a, k, TAU, K,
+                                  dict(unmask=out["unmask"][b], accept=out["accept"][b]))
+    finally:
+        cora.cora_session_destroy(s)
+    print(f"batched replay: {n} steps x {B} sequences, max|dc| = {max_dc:.2e}")
+
+
 def test_denoise_step_rejects_a_wrong_block_or_step(tiny):
     """cora_denoise_step(s, block, step, ...) checks the caller's (block, step)
     against the session before launching: a mismatch is CORA_ESTATE and
