@@ -15,11 +15,15 @@
 //   O += P_j V_j         tcgen05.mma M=128 x N=128 (hd) x K=128 (keys) into one
 //                        TMEM accumulator; V is read as an MN-major operand
 //                        straight from its [keys][hd] layout
-// The reference max m of a row is raised only when a tile's max exceeds it by
-// more than 2^8 (then O and l are rescaled in place, after the previous PV
-// has completed).  The final O / l is the same for any choice of m, and
-// P <= 2^8 keeps full bf16 precision, so the result is unchanged while the
-// softmax warps never wait for a PV in the common case.
+// The reference m of a row is the first tile's max.  Later tiles are
+// exponentiated against it without computing their max; only when a tile's
+// row sum would pass 2^64 (a score more than ~64 above m, in log2 units) is
+// that tile's max taken and m raised to it where it exceeds m by more than 8
+// (then O and l are rescaled in place, after the previous PV has completed)
+// and the tile redone.  The final O / l is the same for any choice of m (bf16
+// and fp32 keep their relative precision at any scale; 2^64 keeps P, l and O
+// far from overflow), so the result is unchanged while the softmax warps skip
+// the max and never wait for a PV in the common case.
 // Two TMEM buffers for S and two P buffers let the softmax of tile j overlap
 // the MMAs of tiles j-1 and j+1.  TMEM: S[0] +0, S[1] +128, O +256.
 // K and V buffers are released separately (K_j once QK_j is done, V_j once
@@ -45,6 +49,7 @@ struct Tile {
   static constexpr int SMEM = 5 * OPND + 4 * COL + 1024 + 256;
 };
 constexpr float kRescale = 8.0f; // log2 headroom before the reference max is raised
+constexpr float kSumLimit = 0x1p64f;  // row sum of a tile beyond which m is raised
 }  // namespace attn
 
 // MN-major (N contiguous) 128-byte-swizzled operand: 8-row K groups 1024 B
@@ -257,63 +262,78 @@ __global__ void __launch_bounds__(192, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&sfree[s]);  // S buffer may take S_{j+2}
       const int kbase = j * KT;
-      float mx8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) mx8[i] = -INFINITY;
       if (kbase + KT > S) {  // ragged last tile: keys past the end do not count
 #pragma unroll
         for (int i = 0; i < KT; ++i)
           if (kbase + i >= S) v[i] = __float_as_uint(-INFINITY);
       }
+      // Exact tile max; raise m where it exceeds m + kRescale (rescaling O
+      // after the previous PV).  Returns false on a timed-out wait.
+      auto raise_to_max = [&]() -> bool {
+        float mx8[8];
 #pragma unroll
-      for (int i = 0; i < KT; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(v[i]));  // eight chains
-      float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                       fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-      mx *= sl2;
-      const bool raise = mx > m + kRescale;
-      if (__any_sync(0xffffffffu, raise)) {
-        const float m_new = raise ? mx : m;
-        const float a = ex2f(m - m_new);  // 0 on the first tile, 1 where not raised
-        l *= a;
-        m = m_new;
-        if (j > 0) {
-          // O holds PV_0 .. PV_{j-1}: wait for the last one, then rescale in place.
-          const int sp = (j - 1) & 1;
-          ok = mbar_wait(&pdone[sp], ((j - 1) >> 1) & 1, abort_flag, err, CORA_DERR_EPI_WAIT);
-          if (!ok) break;
-          tc_fence_after();
+        for (int i = 0; i < 8; ++i) mx8[i] = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < KT; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(v[i]));
+        float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                         fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+        mx *= sl2;
+        const bool raise = mx > m + kRescale;
+        if (__any_sync(0xffffffffu, raise)) {
+          const float m_new = raise ? mx : m;
+          const float a = ex2f(m - m_new);
+          l *= a;
+          m = m_new;
+          if (j > 0) {
+            const int sp = (j - 1) & 1;
+            if (!mbar_wait(&pdone[sp], ((j - 1) >> 1) & 1, abort_flag, err, CORA_DERR_EPI_WAIT)) return false;
+            tc_fence_after();
 #pragma unroll 1
-          for (int c = 0; c < HD; c += 32) {
-            uint32_t o[32];
-            tmem_ld32w(o_lane + c, o);
+            for (int c = 0; c < HD; c += 32) {
+              uint32_t o[32];
+              tmem_ld32w(o_lane + c, o);
 #pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * a);
-            tmem_st32(o_lane + c, o);
+              for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * a);
+              tmem_st32(o_lane + c, o);
+            }
+            tmem_wait_st();
           }
-          tmem_wait_st();
         }
+        return true;
+      };
+      uint8_t* prow = sP[s];
+      auto exp_tile = [&]() -> float {
+        float rs4[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < KT; c += 8) {
+          uint32_t pk[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const float x0 = ex2f(fmaf(__uint_as_float(v[c + 2 * i]), sl2, -m));
+            const float x1 = ex2f(fmaf(__uint_as_float(v[c + 2 * i + 1]), sl2, -m));
+            rs4[i] += x0 + x1;
+            pk[i] = pack_bf16x2(x0, x1);
+          }
+          const int chunk = (c & 63) >> 3;
+          *reinterpret_cast<uint4*>(prow + (c >> 6) * COL + r * 128 + ((chunk ^ (r & 7)) << 4)) =
+              make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        }
+        return (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
+      };
+      if (j == 0) {
+        ok = raise_to_max();
+        if (!ok) break;
       }
       // P buffer s is free once PV_{j-2} has read it.
       if (j >= 2) ok = mbar_wait(&pdone[s], ph ^ 1u, abort_flag, err, CORA_DERR_EPI_WAIT);
       if (!ok) break;
-      float rs4[4] = {0.f, 0.f, 0.f, 0.f};
-      uint8_t* prow = sP[s];
-#pragma unroll
-      for (int c = 0; c < KT; c += 8) {
-        uint32_t pk[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float x0 = ex2f(fmaf(__uint_as_float(v[c + 2 * i]), sl2, -m));
-          const float x1 = ex2f(fmaf(__uint_as_float(v[c + 2 * i + 1]), sl2, -m));
-          rs4[i] += x0 + x1;
-          pk[i] = pack_bf16x2(x0, x1);
-        }
-        // keys c .. c+7 -> swizzle column c/64, 16-byte chunk (c%64)/8
-        const int chunk = (c & 63) >> 3;
-        *reinterpret_cast<uint4*>(prow + (c >> 6) * COL + r * 128 + ((chunk ^ (r & 7)) << 4)) =
-            make_uint4(pk[0], pk[1], pk[2], pk[3]);
+      float rs = exp_tile();
+      if (j > 0 && __any_sync(0xffffffffu, !(rs <= kSumLimit))) {
+        ok = raise_to_max();
+        if (!ok) break;
+        rs = exp_tile();
       }
-      l += (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
+      l += rs;
       fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();

@@ -19,8 +19,11 @@
 // issue order, so QK_g(j+1) overwrites S_g only after PV_g(j) has read P_g(j)
 // from it, and the commit after QK_g(j+1) (the softmax's "S ready" signal)
 // also means PV_g(j) is complete: O_g may then be rescaled in place.  The
-// reference max m of a row is raised only when a tile's max exceeds it by more
-// than 2^8 (then O and l are rescaled); O / l is the same for any m.
+// reference m of a row is the item's first key tile's max; later tiles are
+// exponentiated against it without computing their max, and only when a
+// tile's row sum would pass 2^64 is its max taken, m raised where it exceeds
+// m by more than 8 (O and l rescaled) and the tile redone.  O / l is the same
+// for any m (see attention_tc.cu).
 
 // TMEM: S_0 +0, S_1 +128, O_0 +256, O_1 +384 (512 columns).
 // Shared memory: Q_0, Q_1, K[2], V[2] (32 KB each).  The output O / l goes from
@@ -45,6 +48,7 @@ constexpr int OPND = QT * HD * 2;  // 32 KB: one 128 x 128 bf16 operand (two 16 
 constexpr int SMEM = 6 * OPND + 1024 + 256;  // Q[2], K[2], V[2]
 constexpr int THREADS = 384;
 constexpr float kRescale = 8.0f;   // log2 headroom before the reference max is raised
+constexpr float kSumLimit = 0x1p64f;  // row sum of a tile beyond which m is raised
 }  // namespace attn2
 
 // MN-major (N contiguous) 128-byte-swizzled operand: 8-row K groups 1024 B
@@ -318,47 +322,64 @@ __global__ void __launch_bounds__(attn2::THREADS, 1)
           for (int i = 0; i < KT; ++i)
             if (kbase + i >= S) v[i] = __float_as_uint(-INFINITY);
         }
-        float mx8[8];
+        // P = exp2(S * sl2 - m) as bf16 pairs over the first 64 columns of S_g;
+        // returns the row sum of this tile.
+        auto exp_tile = [&]() -> float {
+          float rs4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int i = 0; i < 8; ++i) mx8[i] = __uint_as_float(v[i]);
+          for (int half = 0; half < 2; ++half) {
+            uint32_t pk[32];
 #pragma unroll
-        for (int i = 8; i < KT; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(v[i]));  // eight chains
-        float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                         fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-        mx *= sl2;
-        const bool raise = mx > m + kRescale;
-        if (__any_sync(0xffffffffu, raise)) {
-          const float m_new = raise ? mx : m;
-          const float a = ex2_approx_ftz(m - m_new);  // 0 on the first tile, 1 where not raised
-          l *= a;
-          m = m_new;
-          if (j > 0) {
-            // O_g holds PV_g up to the previous tile, complete (see above).
+            for (int i = 0; i < 32; ++i) {
+              const float x0 = ex2_approx_ftz(fmaf(__uint_as_float(v[64 * half + 2 * i]), sl2, -m));
+              const float x1 = ex2_approx_ftz(fmaf(__uint_as_float(v[64 * half + 2 * i + 1]), sl2, -m));
+              rs4[i & 3] += x0 + x1;
+              pk[i] = pack_bf16x2(x0, x1);
+            }
+            tm_st32(s_lane + 32 * half, pk);
+          }
+          return (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
+        };
+        // Exact tile max; raise m where it exceeds m + kRescale (rescaling O).
+        auto raise_to_max = [&]() {
+          float mx8[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) mx8[i] = __uint_as_float(v[i]);
+#pragma unroll
+          for (int i = 8; i < KT; ++i) mx8[i & 7] = fmaxf(mx8[i & 7], __uint_as_float(v[i]));
+          float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                           fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+          mx *= sl2;
+          const bool raise = mx > m + kRescale;
+          if (__any_sync(0xffffffffu, raise)) {
+            const float m_new = raise ? mx : m;
+            const float a = ex2_approx_ftz(m - m_new);
+            l *= a;
+            m = m_new;
+            if (j > 0) {
 #pragma unroll 1
-            for (int c = 0; c < HD; c += 32) {
-              uint32_t o[32];
-              tm_ld32(o_lane + c, o);
+              for (int c = 0; c < HD; c += 32) {
+                uint32_t o[32];
+                tm_ld32(o_lane + c, o);
 #pragma unroll
-              for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * a);
-              tm_st32(o_lane + c, o);
+                for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * a);
+                tm_st32(o_lane + c, o);
+              }
             }
           }
-        }
-        // P = exp2(S * sl2 - m) as bf16 pairs over the first 64 columns of S_g.
-        float rs4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          uint32_t pk[32];
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float x0 = ex2_approx_ftz(fmaf(__uint_as_float(v[64 * half + 2 * i]), sl2, -m));
-            const float x1 = ex2_approx_ftz(fmaf(__uint_as_float(v[64 * half + 2 * i + 1]), sl2, -m));
-            rs4[i & 3] += x0 + x1;
-            pk[i] = pack_bf16x2(x0, x1);
+        };
+        float rs;
+        if (j == 0) {
+          raise_to_max();
+          rs = exp_tile();
+        } else {
+          rs = exp_tile();
+          if (__any_sync(0xffffffffu, !(rs <= kSumLimit))) {
+            raise_to_max();
+            rs = exp_tile();
           }
-          tm_st32(s_lane + 32 * half, pk);
         }
-        l += (rs4[0] + rs4[1]) + (rs4[2] + rs4[3]);
+        l += rs;
         tm_wait_st();
         tc_fence_before();
         __syncwarp();

@@ -182,6 +182,35 @@ def test_attention(B, S, Hq, Hkv, hd):
     assert np.abs(got - ref).max() <= atol + 1e-2 * np.abs(ref).max()
 
 
+# Scores that jump far above everything seen earlier in a row: every even
+# query row of every head is 2u (u a random +-1 vector), keys 40, 300 and S-1
+# are 3u, 4u and 8u, so after the 1/sqrt(hd) scale those rows' scores rise by
+# ~98, ~131 and ~261 (log2 units, hd 128) over the first keys' ~N(0, 1): the softmax
+# reference must be raised inside the first key tile and in the last one
+# (where O is rescaled).  One CTA per item (first and last case) and two
+# query tiles per CTA (items > SMs); the last key tile is ragged.
+@pytest.mark.parametrize("B,S,Hq,hd", [(1, 600, 2, 128), (2, 1000, 96, 128), (1, 300, 2, 64)])
+def test_attention_score_jumps(B, S, Hq, hd):
+    Hkv = Hq
+    x = f64(bits(6, 13, (B, S, 3 * Hq, hd), 0.3))
+    rng = np.random.default_rng(7)
+    for b in range(B):
+        for h in range(Hq):
+            u = rng.choice([-1.0, 1.0], size=hd)
+            x[b, 0::2, h] = 2.0 * u
+            for key, scale in ((40, 3.0), (300 % S, 4.0), (S - 1, 8.0)):
+                x[b, key, Hq + h] = scale * u
+    qkv = (x.astype(np.float32).view(np.uint32) >> 16).astype(np.uint16)  # exact: every value is bf16
+    assert np.array_equal(f64(qkv), x)
+    out = torch.zeros((B * S, Hq * hd), dtype=torch.int16, device="cuda")
+    cora.cora_op_attention(dev(qkv.reshape(B * S, 3 * Hq * hd)), out, B, S, Hq, Hkv, hd)
+    ref = np.stack([O.attention(x[b, :, :Hq], x[b, :, Hq: 2 * Hq], x[b, :, 2 * Hq:]) for b in range(B)])
+    got = from_dev_bf16(out).reshape(B, S, Hq, hd)
+    assert np.all(np.isfinite(got))
+    atol = 1e-2 * np.sqrt(np.mean(ref ** 2))
+    assert np.abs(got - ref).max() <= atol + 1e-2 * np.abs(ref).max()
+
+
 # Queries from an offset on (the rows a prefix-cache pass recomputes) against
 # every key, with enough (sequence, head, query tile) items to run the
 # persistent kernel (more items than SMs: 256, 320 and 448 here), a query
@@ -224,7 +253,7 @@ def test_lm_head_top1(R, V, d):
 
 
 # --------------------------------------------------- Eq. 1 from logits
-@pytest.mark.parametrize("rows,V", [(64, 126464), (7, 1000), (3, 1001), (1, 1)])
+@pytest.mark.parametrize("rows,V", [(64, 126464), (1, 126464), (300, 20000), (7, 1000), (3, 1001), (1, 1)])
 def test_reduce_top1(rows, V):
     hist = synth.gate_history(5, 1, rows, V)
     lg = synth.gate_logits_bf16(5, 1, rows, V, hist[-1]).reshape(rows, V)
