@@ -1268,7 +1268,17 @@ constexpr int kRasterGroup = 8;
 // side by side (pair p and p + G/2), and there are too few whole tiles per
 // pair to hide a fix-up of up to four partials behind (measured slower).
 static int gemm2_pairs(int M, int N, int K, int num_sms, GemmEpilogue& ep) {
-  const int pairs = gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2, ep);
+  int pairs = gemm_grid(M > 128 ? (M + 1) / 2 : M, N, K, 256, num_sms / 2, ep);
+  if (ep.splits > 2 && (ep.mode == CORA_EPI_STORE_BF16 || ep.mode == CORA_EPI_RESID_F32)) {
+    // Few pair-tiles (one row block): two pieces sharing the fix-up rather
+    // than three or four skewed ones, whose finisher adds three partials.
+    const int tiles = pairs / ep.splits;
+    ep.splits = 2;
+    ep.split_skew = 0;
+    ep.split_pair = 1;
+    ep.sk_units = tiles * 2;
+    pairs = tiles * 2;
+  }
   const int num_m = (M + 255) / 256;
   const int tiles = num_m * (N / 256);
   if (ep.splits == 0 && num_m > 2 && tiles >= pairs) {
