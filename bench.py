@@ -43,17 +43,21 @@ import numpy as np  # noqa: E402
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM bytes (read + write) per launch from one ncu capture of each kernel on
-# a workload's per-launch shapes (2-layer model), keyed by a hash of the
-# kernel source at capture time and by the workload; null once the source
-# changed, and for workloads without a capture.
+# a workload's per-launch shapes, keyed by a hash of the kernel source at
+# capture time and by the workload; null once the source changed, and for
+# workloads without a capture.
 NCU_TRAFFIC = {
-    # gemm_tc2_kernel, mean of the QKV / O / gate-up / down launches (read + write):
-    # (125.2 + 46.3 + 245.6 + 125.9) MB / 4
-    ("gemm", "9840a7e7c917", "llada8b-shape-256+256"): 135_742_528,
-    # (95.3 + 113.8 + 699.2 + 679.7) MB / 4
-    ("gemm", "9840a7e7c917", "dream7b-shape-256+512-b4"): 397_012_736,
-    # (1049.4 + 631.8 + 1667.1 + 1855.9) MB / 4
-    ("gemm", "9840a7e7c917", "llada8b-shape-512+1024-b8"): 1_301_025_792,
+    # gemm_tc2_kernel, mean of the QKV / O / gate-up / down launches (read + write), from
+    # `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` over the GEMM-alone leg
+    # (`bench.py --gemm-shapes-only WORKLOAD --gemm-reps 1`, the QKV launch with a plain bf16
+    # store), one launch per projection (ncu flushes the caches before every profiled launch; the
+    # four launches of a projection read within 0.5 % of each other):
+    # (112.2 + 9.5 + 46.2 + 0.0 + 218.3 + 24.4 + 121.8 + 0.6) MB / 4
+    ("gemm", "6b8ed2116b11", "llada8b-shape-256+256"): 133_209_856,
+    # (69.8 + 23.5 + 99.3 + 12.3 + 567.6 + 126.2 + 642.1 + 39.2) MB / 4
+    ("gemm", "6b8ed2116b11", "dream7b-shape-256+512-b4"): 394_803_648,
+    # (719.5 + 300.0 + 453.3 + 168.0 + 1320.9 + 310.5 + 1620.7 + 191.3) MB / 4
+    ("gemm", "6b8ed2116b11", "llada8b-shape-512+1024-b8"): 1_270_657_856,
 }
 
 
