@@ -98,7 +98,8 @@ def test_gemm_store(M, N, K):
     close_bf16(from_dev_bf16(Ct), f64(A) @ f64(Bm).T)
 
 
-@pytest.mark.parametrize("M,N,K", [(512, 4096, 4096),    # 32 pair-tiles: two skewed k-splits each
+@pytest.mark.parametrize("M,N,K", [(512, 4096, 4096),    # 32 pair-tiles: two k-pieces sharing the fix-up
+                                   (96, 4096, 12288),    # 1-CTA: four skewed k-pieces, three partials per finisher
                                    (512, 12288, 4096),   # 96 pair-tiles over the SM pairs: stream-K
                                    (2048, 12288, 1024)])  # 384 pair-tiles: stream-K + data-parallel waves
 def test_gemm_split_tiles_are_deterministic(M, N, K):
@@ -111,6 +112,9 @@ def test_gemm_split_tiles_are_deterministic(M, N, K):
 
 @pytest.mark.parametrize("M,N,K", [(300, 512, 320), (130, 256, 1024), (512, 4096, 12288), (100, 16384, 512),
                                    (40, 4096, 12288), (64, 16384, 512),
+                                   (256, 4096, 4096),    # one row block of 16 pair-tiles: two pieces sharing the fix-up
+                                   (96, 4096, 4096),     # 1-CTA, 16 tiles: two pieces sharing the fix-up
+                                   (96, 4096, 12288),    # 1-CTA, 16 tiles, K of 192 k-blocks: four skewed pieces
                                    (1536, 8192, 512)])  # 192 pair-tiles: stream-K + one data-parallel wave
 def test_gemm_residual(M, N, K):
     A = bits(3, 10, (M, K), 1.0)
