@@ -470,7 +470,16 @@ __global__ void step_loop_cond_kernel(cudaGraphConditionalHandle h, int32_t* sta
 using namespace cora;
 
 int reduce_top1_parts_count(int rows, int V, int num_sms) {
+  // Resident 256-thread CTAs per SM (register-limited), looked up once.
+  static int per_sm = 0;
+  if (per_sm == 0) {
+    int b = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&b, reduce_fused_kernel, 256, 0) != cudaSuccess || b < 1) b = 4;
+    per_sm = b;
+  }
   int want = (4 * num_sms + rows - 1) / rows;    // about four CTAs per SM in total (one wave)
+  const int fit = per_sm * num_sms / rows;       // chunks per row that still run in one wave
+  if (fit >= 1 && want > fit) want = fit;        // (8 x 32 rows: 3 chunks = 768 CTAs > 760 slots)
   int max_chunks = (V + 4095) / 4096;            // at least 4096 elements per CTA
   int n = want < max_chunks ? want : max_chunks;
   return n < 1 ? 1 : n;
