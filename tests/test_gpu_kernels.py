@@ -89,6 +89,7 @@ def run_gemm(A, Bm, M, N, K, epi, out_cols, out_dtype=torch.int16, C0=None, **kw
                                    (96, 768, 256), (1, 256, 128), (512, 4096, 4096), (512, 12288, 1024),
                                    (96, 768, 2048), (128, 16384, 512),
                                    (64, 12288, 1024), (16, 4096, 4096), (5, 384, 640),    # few-row kernel
+                                   (256, 12288, 1024),   # one row block, 48 pair-tiles: whole tiles on 48 pairs
                                    (2048, 12288, 256),   # 384 pair-tiles: stream-K + 4 data-parallel waves
                                    (1800, 10240, 192)])  # 320 pair-tiles, ragged last row block, 3 waves
 def test_gemm_store(M, N, K):
@@ -147,7 +148,8 @@ def rope_table(seq, hd, theta):
 
 @pytest.mark.parametrize("B,S,H,Hkv,hd,theta", [(2, 96, 4, 4, 64, 1e4), (1, 300, 2, 1, 128, 5e5),
                                                   (1, 96, 4, 4, 64, 1e4), (1, 100, 2, 1, 128, 5e5),
-                                                  (1, 48, 4, 4, 64, 1e4), (1, 60, 2, 1, 128, 5e5)])
+                                                  (1, 48, 4, 4, 64, 1e4), (1, 60, 2, 1, 128, 5e5),
+                                                  (1, 224, 32, 8, 128, 5e5)])  # one row block, 24 whole pair-tiles
 def test_gemm_rope(B, S, H, Hkv, hd, theta):
     d = 256
     N = (H + 2 * Hkv) * hd
