@@ -51,14 +51,15 @@ NCU_TRAFFIC = {
     # `ncu --metrics dram__bytes_read.sum,dram__bytes_write.sum` over the GEMM-alone leg
     # (`bench.py --gemm-shapes-only WORKLOAD --gemm-reps 1`, the QKV launch with a plain bf16
     # store), one launch per projection (ncu flushes the caches before every profiled launch; the
-    # four launches of a projection read within 0.5 % of each other; later host-side rules for
-    # launches of one row block (at most 256 rows), none of these, left the capture valid):
-    # (112.2 + 9.5 + 46.2 + 0.0 + 218.3 + 24.4 + 121.8 + 0.6) MB / 4
-    ("gemm", "ee42056bbf56", "llada8b-shape-256+256"): 133_209_856,
+    # four launches of a projection read within 0.5 % of each other; the 256 + 256 line was
+    # re-captured after the 512-row gate/up launch moved to data-parallel waves, and the rules for
+    # launches of at most 256 rows, none of these, left the other two valid):
+    # (112.0 + 9.6 + 46.2 + 0.0 + 215.3 + 24.2 + 121.8 + 0.6) MB / 4 (the gate/up launch in data-parallel waves)
+    ("gemm", "1e032d16cd9e", "llada8b-shape-256+256"): 132_433_152,
     # (69.8 + 23.5 + 99.3 + 12.3 + 567.6 + 126.2 + 642.1 + 39.2) MB / 4
-    ("gemm", "ee42056bbf56", "dream7b-shape-256+512-b4"): 394_803_648,
+    ("gemm", "1e032d16cd9e", "dream7b-shape-256+512-b4"): 394_803_648,
     # (719.5 + 300.0 + 453.3 + 168.0 + 1320.9 + 310.5 + 1620.7 + 191.3) MB / 4
-    ("gemm", "ee42056bbf56", "llada8b-shape-512+1024-b8"): 1_270_657_856,
+    ("gemm", "1e032d16cd9e", "llada8b-shape-512+1024-b8"): 1_270_657_856,
 }
 
 
