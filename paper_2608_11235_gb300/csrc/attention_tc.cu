@@ -327,6 +327,8 @@ __global__ void __launch_bounds__(192, 1)
       // P buffer s is free once PV_{j-2} has read it.
       if (j >= 2) ok = mbar_wait(&pdone[s], ph ^ 1u, abort_flag, err, CORA_DERR_EPI_WAIT);
       if (!ok) break;
+      // Later tiles are exponentiated against m without their own max; only
+      // when a row's sum would pass kSumLimit is the max taken and the tile redone.
       float rs = exp_tile();
       if (j > 0 && __any_sync(0xffffffffu, !(rs <= kSumLimit))) {
         ok = raise_to_max();

@@ -373,6 +373,8 @@ __global__ void __launch_bounds__(attn2::THREADS, 1)
           raise_to_max();
           rs = exp_tile();
         } else {
+          // Against m without this tile's max; redone with it only when a row's
+          // sum would pass kSumLimit.
           rs = exp_tile();
           if (__any_sync(0xffffffffu, !(rs <= kSumLimit))) {
             raise_to_max();
