@@ -53,13 +53,14 @@ NCU_TRAFFIC = {
     # store), one launch per projection (ncu flushes the caches before every profiled launch; the
     # four launches of a projection read within 0.5 % of each other; the 256 + 256 line was
     # re-captured after the 512-row gate/up launch moved to data-parallel waves, and the rules for
-    # launches of at most 256 rows, none of these, left the other two valid):
+    # launches of at most 256 rows, none of these, left the other two valid; so did making the
+    # work-split helpers callable from the host for cora_gemm_plan, which left the device code as it was):
     # (112.0 + 9.6 + 46.2 + 0.0 + 215.3 + 24.2 + 121.8 + 0.6) MB / 4 (the gate/up launch in data-parallel waves)
-    ("gemm", "1e032d16cd9e", "llada8b-shape-256+256"): 132_433_152,
+    ("gemm", "56665881d5de", "llada8b-shape-256+256"): 132_433_152,
     # (69.8 + 23.5 + 99.3 + 12.3 + 567.6 + 126.2 + 642.1 + 39.2) MB / 4
-    ("gemm", "1e032d16cd9e", "dream7b-shape-256+512-b4"): 394_803_648,
+    ("gemm", "56665881d5de", "dream7b-shape-256+512-b4"): 394_803_648,
     # (719.5 + 300.0 + 453.3 + 168.0 + 1320.9 + 310.5 + 1620.7 + 191.3) MB / 4
-    ("gemm", "1e032d16cd9e", "llada8b-shape-512+1024-b8"): 1_270_657_856,
+    ("gemm", "56665881d5de", "llada8b-shape-512+1024-b8"): 1_270_657_856,
 }
 
 

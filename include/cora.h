@@ -409,6 +409,24 @@ CORA_API int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32_t
                  int32_t epilogue, const float* rope, int32_t seq, int32_t head_dim, int32_t rope_cols,
                  void* stream);
 
+/* How cora_op_gemm (and the dense pass) divides an M x N x K GEMM with the
+ * given epilogue among CTAs on a GPU with num_sms SMs, computed on the host
+ * with the same rules and the same segment walk the kernels use; no device
+ * work, no CUDA call (usable without a GPU).  A test aid for the work split;
+ * the paper has no counterpart.
+ *   info  int32 [7], written: kernel (0 few-row, 1 one CTA per 128-row tile,
+ *         2 CTA pairs on 256-row tiles), units (CTAs or CTA pairs), tiles,
+ *         k-blocks per tile (K / 64), k-pieces per split tile (0: stream-K or
+ *         whole tiles), 1 when two pieces share the fix-up, data-parallel waves
+ *   seg   int32 [cap][6], written up to cap rows: unit, tile, first k-block,
+ *         end k-block, row block, column block, in each unit's visiting order
+ *         (kernel 0 has no segments)
+ *   n_seg int32 [1], written: the number of segments (may exceed cap)
+ * Errors: CORA_EINVAL for NULL pointers, M < 1, num_sms < 2, K % 64 != 0,
+ * N % 128 != 0 or cap < 0. */
+CORA_API int cora_gemm_plan(int32_t M, int32_t N, int32_t K, int32_t epilogue, int32_t num_sms, int32_t* info,
+                            int32_t* seg, int32_t cap, int32_t* n_seg);
+
 /* Non-causal attention of B sequences of length S from a fused QKV buffer
  * qkv bf16 [B*S, (Hq + 2*Hkv)*hd] (Q heads, then K heads, then V heads;
  * RoPE already applied) into out bf16 [B*S, Hq*hd]; softmax(QK^T/sqrt(hd))V,

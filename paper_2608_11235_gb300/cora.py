@@ -27,7 +27,7 @@ EXPORTED = [
     "cora_op_gemm", "cora_op_attention", "cora_op_rmsnorm", "cora_op_lm_head_top1", "cora_synth_normal_bf16",
     "cora_device_error", "cora_session_profile_step", "cora_session_stream", "cora_reduce_top1_noalloc",
     "cora_session_create_ex", "cora_generate_ex", "cora_session_disagreement", "cora_check_wait_timeout",
-    "cora_session_finished", "cora_op_attention_rows",
+    "cora_session_finished", "cora_op_attention_rows", "cora_gemm_plan",
 ]
 DTYPE_BF16, DTYPE_F32 = 0, 1
 SCHEDULE_FIXED, SCHEDULE_REMAINING = 0, 1
@@ -107,6 +107,7 @@ def lib():
             "cora_reduce_top1_noalloc": ([vp, i32, i32, vp, vp, vp], C.c_int),
             "cora_reduce_gate": ([vp, i32, i32, i32] + [vp] * 6 + [i32, f32, i32] + [vp] * 3 + [vp], C.c_int),
             "cora_op_gemm": ([vp, vp, vp, i32, i32, i32, i32, i32, vp, i32, i32, i32, vp], C.c_int),
+            "cora_gemm_plan": ([i32, i32, i32, i32, i32, vp, vp, i32, vp], C.c_int),
             "cora_op_attention": ([vp, vp, i32, i32, i32, i32, i32, vp], C.c_int),
             "cora_op_attention_rows": ([vp, vp, i32, i32, i32, i32, i32, i32, i32, vp], C.c_int),
             "cora_op_rmsnorm": ([vp, vp, vp, i32, i32, f32, vp], C.c_int),
@@ -330,6 +331,19 @@ def cora_reduce_gate(logits, B, R, V, conf, argmax, prev, persist, state, tokens
     _check("cora_reduce_gate", lib().cora_reduce_gate(
         ptr(logits), B, R, V, ptr(conf), ptr(argmax), ptr(prev), ptr(persist), ptr(state), ptr(tokens), k, tau, K,
         ptr(unmask), ptr(accept), ptr(done), _stream(stream)))
+
+
+def cora_gemm_plan(M: int, N: int, K: int, epilogue: int, num_sms: int):
+    """Host-side work split of a GEMM (cora_gemm_plan): (info dict, segments [n, 6] int32 array of
+    unit, tile, kb0, kb1, row block, column block in each unit's visiting order)."""
+    info = np.zeros(7, np.int32)
+    n = np.zeros(1, np.int32)
+    _check("cora_gemm_plan", lib().cora_gemm_plan(M, N, K, epilogue, num_sms, ptr(info), None, 0, ptr(n)))
+    seg = np.zeros((max(int(n[0]), 1), 6), np.int32)
+    _check("cora_gemm_plan", lib().cora_gemm_plan(M, N, K, epilogue, num_sms, ptr(info), ptr(seg), int(n[0]),
+                                                  ptr(n)))
+    keys = ("kernel", "units", "tiles", "kb", "splits", "split_pair", "dp_waves")
+    return dict(zip(keys, (int(x) for x in info))), seg[: int(n[0])]
 
 
 def cora_op_gemm(A, B, Cm, M, N, K, ldc, epilogue, rope=None, seq=0, head_dim=0, rope_cols=0, stream=None) -> None:

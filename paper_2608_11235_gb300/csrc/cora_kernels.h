@@ -179,6 +179,9 @@ bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t
 int gemm_block_n(int N, int mode);
 // Failure-detection self-check (see cora_check_wait_timeout).
 cudaError_t launch_wait_check(int which, const int* flag, int* err, cudaStream_t st);
+// Host-side plan of launch_gemm's work split (see cora_gemm_plan); returns the
+// number of segments, writes info[7] and up to cap segments of 6 ints.
+int gemm_plan(int M, int N, int K, int mode, int num_sms, int* info, int* seg, int cap);
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M, int N, int K,
                         const GemmEpilogue& ep, const GemmWorkspace& ws, int* err, int num_sms, cudaStream_t st);
 bool make_gemm_out_tmap(CUtensorMap* map, void* C, int M, int ldc, int mode);

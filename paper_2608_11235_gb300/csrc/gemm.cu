@@ -74,7 +74,7 @@ struct WorkSplit {
   // Whole tiles each of the P units runs after its stream-K range: unit c
   // runs tile W / KB + w P + c in wave w.
   int dp_waves, P;
-  __device__ int start(int c) const {
+  __host__ __device__ int start(int c) const {
     if (skew > 0) {
       const int t = c / S, s = c - t * S;
       return t * KB + (s == 0 ? 0 : KB - (S - s) * (KB / S - skew));
@@ -91,7 +91,7 @@ struct WorkSplit {
 // whole tiles.
 struct SegIter {
   int it0, it1, kb_per_tile, t_first, t_last, idx, n_sk, dp_t0, dp_stride, dp_n;
-  __device__ SegIter(int c, const WorkSplit& ws)
+  __host__ __device__ SegIter(int c, const WorkSplit& ws)
       : it0(c < ws.G ? ws.start(c) : ws.W), it1(c < ws.G ? ws.start(c + 1) : ws.W), kb_per_tile(ws.KB), idx(0) {
     t_first = it0 / ws.KB;
     t_last = it1 > it0 ? (it1 - 1) / ws.KB : t_first - 1;
@@ -100,7 +100,7 @@ struct SegIter {
     dp_stride = ws.P;
     dp_n = ws.dp_waves;
   }
-  __device__ bool next(int& t, int& kb0, int& kb1) {
+  __host__ __device__ bool next(int& t, int& kb0, int& kb1) {
     const int KB = kb_per_tile;
     if (idx >= n_sk) {  // data-parallel whole tiles
       const int w = idx - n_sk;
@@ -132,14 +132,14 @@ struct SegIter {
     return true;
   }
   // True once the segment just returned is the last one this CTA visits.
-  __device__ bool finished() const { return idx >= n_sk + dp_n; }
+  __host__ __device__ bool finished() const { return idx >= n_sk + dp_n; }
 };
 
 // Row block and column block of tile t: tiles are numbered in groups of
 // `group` row blocks (the last group may be smaller), row block fastest
 // within a group, so consecutive tiles share weight tiles (B) and the group's
 // row blocks (A) stay in L2 while its columns are walked.  group = 1: M-slowest.
-__device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group, int& mb, int& nb) {
+__host__ __device__ __forceinline__ void tile_coords(int t, int num_m, int num_n, int group, int& mb, int& nb) {
   const int per_group = group * num_n;
   const int g = t / per_group, r = t - g * per_group;
   const int gm = min(group, num_m - g * group);
@@ -1243,18 +1243,14 @@ static int gemm_grid(int M, int N, int K, int bn, int num_sms, GemmEpilogue& ep)
   return ep.sk_units;
 }
 
-template <int BN>
-static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M,
-                                  int N, int K, const GemmEpilogue& ep, const GemmWorkspace& ws, int* err,
-                                  int num_sms, cudaStream_t st) {
-  using Cfg = GemmCfg<BN>;
-  GemmEpilogue e = ep;
-  int grid = gemm_grid(M, N, K, BN, num_sms, e);
+// Grid of the 1-CTA kernel: gemm_grid, then two pieces sharing the fix-up
+// instead of three or four skewed ones (whose finisher adds three partials),
+// unless K is so long that half of it outweighs that: measured at 80-128 rows,
+// O (K = 4096) 23.8-24.7 -> 16.6-17.6 us, down (K = 12288) 43.1-43.7 ->
+// 45.4-45.9 us.
+static int gemm1_grid(int M, int N, int K, int bn, int num_sms, GemmEpilogue& e) {
+  int grid = gemm_grid(M, N, K, bn, num_sms, e);
   if (e.splits > 2 && K / kBK <= kPairMaxKb1 && (e.mode == CORA_EPI_STORE_BF16 || e.mode == CORA_EPI_RESID_F32)) {
-    // Two pieces sharing the fix-up instead of three or four skewed ones
-    // (whose finisher adds three partials), unless K is so long that half of
-    // it outweighs that: measured at 80-128 rows, O (K = 4096) 23.8-24.7 ->
-    // 16.6-17.6 us, down (K = 12288) 43.1-43.7 -> 45.4-45.9 us.
     const int tiles = grid / e.splits;
     e.splits = 2;
     e.split_skew = 0;
@@ -1262,6 +1258,16 @@ static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB
     e.sk_units = tiles * 2;
     grid = tiles * 2;
   }
+  return grid;
+}
+
+template <int BN>
+static cudaError_t launch_gemm_bn(const CUtensorMap& tmA, const CUtensorMap& tmB, const CUtensorMap& tmC, int M,
+                                  int N, int K, const GemmEpilogue& ep, const GemmWorkspace& ws, int* err,
+                                  int num_sms, cudaStream_t st) {
+  using Cfg = GemmCfg<BN>;
+  GemmEpilogue e = ep;
+  const int grid = gemm1_grid(M, N, K, BN, num_sms, e);
   return launch_pdl(gemm_tc_kernel<BN>, dim3(grid), dim3(192), Cfg::SMEM_BYTES, st, tmA, tmB, tmC, M, N, K, e, ws,
                     err);
 }
@@ -1350,6 +1356,72 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, const CU
   if (gemm_block_n(N, ep.mode) == 256)
     return launch_gemm_bn<256>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);
   return launch_gemm_bn<128>(tmA, tmB, tmC, M, N, K, ep, ws, err, num_sms, st);
+}
+
+// Host-side view of how launch_gemm divides an M x N x K projection: the
+// kernel it picks and, for the row-tiled kernels, every unit's (CTA or CTA
+// pair's) segments in visiting order, as the kernels' own SegIter walks them
+// (no device work).  seg: [cap][6] = unit, tile, kb0, kb1, row block, column
+// block.  Returns the number of segments (all of them, even beyond cap).
+int gemm_plan(int M, int N, int K, int mode, int num_sms, int* info, int* seg, int cap) {
+  GemmEpilogue ep{};
+  ep.mode = mode;
+  ep.head_dim = 128;  // (the few-row kernel's RoPE check; every workload here has head_dim 64 or 128)
+  static const uint16_t probe = 0;
+  ep.a_ptr = &probe;  // only its presence matters to the few-row kernel's check
+  int kind, units, num_m, num_n, group = 1, dp = 0;
+  if (gemm_skinny_supported(M, N, K, ep)) {
+    info[0] = 0;
+    for (int i = 1; i < 7; ++i) info[i] = 0;
+    return 0;
+  }
+  const int KB = K / kBK;
+  int W;
+  if (M > 128 && N % 256 == 0 && g_gemm_pairs_enabled) {
+    kind = 2;
+    units = gemm2_pairs(M, N, K, num_sms, ep);
+    num_m = (M + 255) / 256;
+    num_n = N / 256;
+    group = ep.raster_group;
+    dp = ep.dp_waves;
+    W = (num_m * num_n - dp * units) * KB;
+  } else {
+    kind = 1;
+    const int bn = gemm_block_n(N, mode);
+    units = gemm1_grid(M, N, K, bn, num_sms, ep);
+    num_m = (M + kBM - 1) / kBM;
+    num_n = N / bn;
+    W = num_m * num_n * KB;
+    ep.sk_units = units;
+  }
+  info[0] = kind;
+  info[1] = units;
+  info[2] = num_m * num_n;
+  info[3] = KB;
+  info[4] = ep.splits;
+  info[5] = ep.split_pair;
+  info[6] = dp;
+  const WorkSplit ws{ep.sk_units, W, KB, ep.splits, ep.split_skew, dp, units};
+  int n = 0;
+  for (int u = 0; u < units; ++u) {
+    SegIter it(u, ws);
+    int t, kb0, kb1;
+    while (it.next(t, kb0, kb1)) {
+      if (n < cap) {
+        int mb, nb;
+        tile_coords(t, num_m, num_n, group, mb, nb);
+        int* r = seg + 6 * n;
+        r[0] = u;
+        r[1] = t;
+        r[2] = kb0;
+        r[3] = kb1;
+        r[4] = mb;
+        r[5] = nb;
+      }
+      ++n;
+    }
+  }
+  return n;
 }
 
 __global__ void rope_transpose_kernel(const float2* __restrict__ rope, float2* __restrict__ rope_t, int seq, int half) {

@@ -1088,6 +1088,17 @@ extern "C" int cora_reduce_gate(const uint16_t* logits, int32_t B, int32_t R, in
   return CORA_OK;
 }
 
+extern "C" int cora_gemm_plan(int32_t M, int32_t N, int32_t K, int32_t epilogue, int32_t num_sms, int32_t* info,
+                              int32_t* seg, int32_t cap, int32_t* n_seg) {
+  REQUIRE(info && n_seg && (seg || cap == 0), "cora_gemm_plan: NULL pointer");
+  REQUIRE(M >= 1 && num_sms >= 2 && K >= 64 && K % 64 == 0 && N >= 128 && N % 128 == 0 && cap >= 0,
+          "cora_gemm_plan: bad M/N/K/num_sms/cap");
+  REQUIRE(epilogue >= 0 && epilogue <= 3, "cora_gemm_plan: bad epilogue");
+  REQUIRE(epilogue != CORA_EPI_SWIGLU || N % 256 == 0, "cora_gemm_plan: SWIGLU needs N %% 256 == 0");
+  *n_seg = gemm_plan(M, N, K, epilogue, num_sms, info, seg, cap);
+  return CORA_OK;
+}
+
 extern "C" int cora_op_gemm(const uint16_t* A, const uint16_t* B, void* C, int32_t M, int32_t N, int32_t K,
                             int32_t ldc, int32_t epilogue, const float* rope, int32_t seq, int32_t head_dim,
                             int32_t rope_cols, void* stream) {
